@@ -1,0 +1,497 @@
+#!/usr/bin/env python3
+"""Throughput benchmark of the SGD-KV compression step on GB300.
+
+One step = the whole hot path for one model's prefilled cache: the head-level budget
+allocation (host, Eq. 2 + Algorithm 1) and, for every layer, window scoring + max-pool
+(sgdkv_score) and top-b_h selection + K/V gather (sgdkv_compact) over all KV heads.
+Metric: compressed context tokens per second per layer = n_layers * L / step time.
+Inputs are seeded synthetic caches shaped like the paper's models (no datasets/weights).
+
+Prints one JSON line (rank 0).  Also reports the roofline of the dominant kernel stage,
+the end-to-end figure through the C-ABI from pinned host buffers, and the CPU oracle
+timed on this machine's host cores on a bounded sample.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--frac F]
+  python bench.py --impl reference ...   # the CPU oracle as the reference arm
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+DEFAULT_WORKLOAD = "c3_qwen25_7b_L128k"
+METRIC = "compressed context tokens/sec per layer"
+UNIT = "tokens/s/layer"
+
+
+def parse_args(argv=None):
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    p.add_argument("--frac", type=float, default=0.25)
+    p.add_argument("--layers", type=int, default=0, help="layers per step (0 = all)")
+    p.add_argument("--e2e-steps", type=int, default=3)
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-child", action="store_true", help=argparse.SUPPRESS)
+    return p.parse_args(argv)
+
+
+# ------------------------------------------------------------------------------------------
+# multi-process plumbing (one process per GPU; replicas, no data-path collective)
+# ------------------------------------------------------------------------------------------
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def dist_init(world):
+    if world > 1:
+        import torch.distributed as dist
+        if not dist.is_initialized():
+            dist.init_process_group("gloo")
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------------------------------
+# clocks during the timed region
+# ------------------------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str | None):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+            os.close(fd)
+            cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                   "-lms", "100"]
+            if self.gpu_id is not None:
+                cmd += ["-i", self.gpu_id]
+            self.proc = subprocess.Popen(cmd, stdout=open(self.path, "w"),
+                                         stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) != 9:
+                    continue
+                try:
+                    rows.append(dict(sm=float(parts[1]), max=float(parts[2]),
+                                     hw=parts[5], hwt=parts[6], swt=parts[7], swp=parts[8]))
+                except ValueError:
+                    continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        reasons = set()
+        for r in rows:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                              ("swt", "sw_thermal_slowdown"), ("swp", "sw_power_cap")):
+                if r[key].lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(r["sm"] for r in rows),
+                "sm_max_mhz": max(r["max"] for r in rows), "samples": len(rows),
+                "reasons": sorted(reasons)}
+
+
+def nvsmi_id(dev_index: int) -> str | None:
+    try:
+        import torch
+        props = torch.cuda.get_device_properties(dev_index)
+        u = getattr(props, "uuid", None)
+        if u is not None:
+            s = str(u)
+            return s if s.startswith("GPU-") else "GPU-" + s
+    except Exception:
+        pass
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+    ids = [v for v in vis.split(",") if v.strip()]
+    return ids[dev_index] if dev_index < len(ids) else None
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            m = json.load(f)
+        return dict(hbm=float(m["hbm_gbs"]), bf16=float(m["bf16_tflops"]),
+                    bf16_sus=float(m["bf16_tflops_sustained"]), source="measured")
+    except Exception:
+        return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
+
+
+# ------------------------------------------------------------------------------------------
+# algorithmic work (per layer)
+# ------------------------------------------------------------------------------------------
+
+def score_flops(wl) -> float:
+    """Two passes over every (window row, key) pair: 2 * (2 * G * W * d) per key per KV head."""
+    return 2.0 * 2.0 * wl.G * wl.W * wl.d * wl.L * wl.Hkv
+
+
+def path_bytes(wl, budgets_layer) -> float:
+    """K read once (d*2 B/key), score written and read (8 B/key), and per kept row: K and V
+    read and written (4*d*2 B) plus its int32 index."""
+    per_key = wl.d * 2 + 8
+    return float(wl.Hkv * wl.L * per_key + sum(int(b) for b in budgets_layer) * (4 * wl.d * 2 + 4))
+
+
+# ------------------------------------------------------------------------------------------
+# our arm
+# ------------------------------------------------------------------------------------------
+
+def run_ours(args, world, rank, local):
+    import numpy as np
+    import torch
+
+    from paper_2609_03235_gb300 import configs, synth
+    from paper_2609_03235_gb300 import sgdkv as sg
+
+    wl = configs.BY_NAME[args.workload]
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    sg.lib()
+    n_sink, n_recent = configs.sink_recent_split(wl.floor)
+    hs = synth.head_scores(wl)
+    T = wl.total_budget(args.frac)
+    b_all = sg.sgdkv_allocate_budgets(hs, wl.L, T, wl.floor)
+    Ls = wl.n_layers if args.layers <= 0 else min(args.layers, wl.n_layers)
+    layers = [synth.layer_inputs_device(wl, l, dev) for l in range(Ls)]
+    outs = []
+    for l in range(Ls):
+        b = b_all[l * wl.Hkv:(l + 1) * wl.Hkv]
+        tot = int(b.sum())
+        outs.append(dict(
+            b=b, scores=torch.empty((wl.Hkv, wl.L), dtype=torch.float32, device=dev),
+            idx=torch.empty(tot, dtype=torch.int32, device=dev),
+            cu=torch.empty(wl.Hkv + 1, dtype=torch.int32, device=dev),
+            ko=torch.empty((tot, wl.d), dtype=torch.bfloat16, device=dev),
+            vo=torch.empty((tot, wl.d), dtype=torch.bfloat16, device=dev)))
+    ws = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(ev=None):
+        ball = sg.sgdkv_allocate_budgets(hs, wl.L, T, wl.floor)      # a1 (host)
+        for l in range(Ls):
+            inp, o = layers[l], outs[l]
+            b = ball[l * wl.Hkv:(l + 1) * wl.Hkv]
+            if ev is not None:
+                ev[l][0].record(stream)
+            sg.sgdkv_score(inp["q"], inp["K"], wl.W, wl.pool, o["scores"], ws, stream)
+            if ev is not None:
+                ev[l][1].record(stream)
+            sg.sgdkv_compact(inp["K"], inp["V"], o["scores"], b, n_sink, n_recent, o["idx"],
+                             o["cu"], o["ko"], o["vo"], ws, stream)
+
+    for _ in range(max(args.warmup, 0)):
+        step()
+    torch.cuda.synchronize(dev)
+    st = sg.sgdkv_last_error(ws, stream)
+    if st != sg.OK:
+        raise RuntimeError(f"device-side error during warm-up: {sg.status_string(st)}")
+
+    K = args.steps
+    evs = [[[torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)]
+            for _ in range(Ls)] for _ in range(K)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(nvsmi_id(local))
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    clocks.start()
+    time.sleep(0.3)                      # let the sampler attach before the timed region
+    launches0 = sg.sgdkv_launch_count()
+    start.record(stream)
+    for k in range(K):
+        step(evs[k])
+    end.record(stream)
+    torch.cuda.synchronize(dev)
+    launches = sg.sgdkv_launch_count() - launches0
+    clk = clocks.stop()
+    barrier(world)
+    st = sg.sgdkv_last_error(ws, stream)
+    if st != sg.OK:
+        raise RuntimeError(f"device-side error in the timed region: {sg.status_string(st)}")
+    ms = start.elapsed_time(end) / K
+    ms_max = max_over_ranks(ms, world)
+    score_ms = statistics.mean(evs[k][l][0].elapsed_time(evs[k][l][1])
+                               for k in range(K) for l in range(Ls))
+
+    peaks = measured_peaks()
+    flops = score_flops(wl)
+    achieved_tf = flops / (score_ms * 1e-3) / 1e12
+    bytes_step = sum(path_bytes(wl, o["b"]) for o in outs)
+    value = world * wl.L * Ls / (ms_max * 1e-3)
+
+    e2e = None
+    if not args.no_e2e and args.e2e_steps > 0:
+        e2e = run_e2e(args, wl, layers, outs, n_sink, n_recent, dev, world)
+
+    rec = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) K/V/Q with planted sink and salient keys)",
+        "config": {"workload": wl.name, "model_shape": "Qwen2.5-7B-1M" if wl.Hkv == 4 else "Qwen3-32B",
+                   "n_layers": Ls, "Hq": wl.Hq, "Hkv": wl.Hkv, "head_dim": wl.d,
+                   "context_len": wl.L, "window": wl.W, "pool": wl.pool,
+                   "budget_frac": args.frac, "floor": wl.floor, "n_sink": n_sink,
+                   "n_recent": n_recent, "parallelism": f"replicas x{world}",
+                   "l2": "inputs larger than L2 (K+V of one layer = %d MiB)" %
+                         (2 * wl.Hkv * wl.L * wl.d * 2 >> 20)},
+        "roofline": {"kernel": "score stage (sgdkv_score: window logits, softmax sums, pool)",
+                     "bound": "tensor", "achieved": achieved_tf, "peak": peaks["bf16_sus"],
+                     "unit": "TFLOP/s", "frac": achieved_tf / peaks["bf16_sus"],
+                     "traffic": None, "peak_source": peaks["source"] + " bf16 sustained",
+                     "ms_per_launch": score_ms, "flops_per_launch": flops},
+        "hbm_path": {"achieved_gbs": bytes_step / (ms_max * 1e-3) / 1e9,
+                     "peak_gbs": peaks["hbm"], "frac": bytes_step / (ms_max * 1e-3) / 1e9 / peaks["hbm"],
+                     "bytes_per_step": bytes_step},
+        "gpu_launches": int(launches),
+        "clocks": clk,
+        "e2e": e2e,
+    }
+    return rec
+
+
+def run_e2e(args, wl, layers, outs, n_sink, n_recent, dev, world):
+    """Same metric through the public API with host buffers: every step copies each layer's
+    q/K/V from pinned host memory, compresses it, and copies the compressed cache back."""
+    import torch
+
+    from paper_2609_03235_gb300 import sgdkv as sg
+
+    Ls = len(layers)
+    hq = [l["q"].cpu().pin_memory() for l in layers]
+    hk = [l["K"].cpu().pin_memory() for l in layers]
+    hv = [l["V"].cpu().pin_memory() for l in layers]
+    ho = [dict(idx=torch.empty(o["idx"].shape, dtype=torch.int32).pin_memory(),
+               cu=torch.empty(o["cu"].shape, dtype=torch.int32).pin_memory(),
+               ko=torch.empty(o["ko"].shape, dtype=torch.bfloat16).pin_memory(),
+               vo=torch.empty(o["vo"].shape, dtype=torch.bfloat16).pin_memory()) for o in outs]
+    slots = []
+    maxtot = max(o["idx"].numel() for o in outs)
+    for _ in range(2):
+        slots.append(dict(
+            q=torch.empty_like(layers[0]["q"]), K=torch.empty_like(layers[0]["K"]),
+            V=torch.empty_like(layers[0]["V"]),
+            idx=torch.empty(maxtot, dtype=torch.int32, device=dev),
+            cu=torch.empty(wl.Hkv + 1, dtype=torch.int32, device=dev),
+            ko=torch.empty((maxtot, wl.d), dtype=torch.bfloat16, device=dev),
+            vo=torch.empty((maxtot, wl.d), dtype=torch.bfloat16, device=dev),
+            ws=sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)))
+    s_h2d, s_cmp, s_d2h = torch.cuda.Stream(dev), torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    ev = lambda: torch.cuda.Event()
+    h2d_done = [ev(), ev()]
+    cmp_done = [ev(), ev()]
+    d2h_done = [ev(), ev()]
+    hs = None
+    from paper_2609_03235_gb300 import synth
+    hs = synth.head_scores(wl)
+    T = wl.total_budget(args.frac)
+    h2d_bytes = sum(hq[l].numel() * 2 + hk[l].numel() * 2 + hv[l].numel() * 2 for l in range(Ls))
+    d2h_bytes = sum(ho[l]["idx"].numel() * 4 + ho[l]["cu"].numel() * 4 +
+                    ho[l]["ko"].numel() * 2 + ho[l]["vo"].numel() * 2 for l in range(Ls))
+
+    def step():
+        ball = sg.sgdkv_allocate_budgets(hs, wl.L, T, wl.floor)
+        for l in range(Ls):
+            s = l % 2
+            sl = slots[s]
+            b = ball[l * wl.Hkv:(l + 1) * wl.Hkv]
+            tot = int(b.sum())
+            s_h2d.wait_event(cmp_done[s])
+            with torch.cuda.stream(s_h2d):
+                sl["q"].copy_(hq[l], non_blocking=True)
+                sl["K"].copy_(hk[l], non_blocking=True)
+                sl["V"].copy_(hv[l], non_blocking=True)
+                h2d_done[s].record(s_h2d)
+            s_cmp.wait_event(h2d_done[s])
+            s_cmp.wait_event(d2h_done[s])
+            sg.sgdkv_compress_layer(sl["q"], sl["K"], sl["V"], b, wl.W, wl.pool, n_sink,
+                                    n_recent, None, sl["idx"], sl["cu"], sl["ko"], sl["vo"],
+                                    sl["ws"], s_cmp)
+            cmp_done[s].record(s_cmp)
+            s_d2h.wait_event(cmp_done[s])
+            with torch.cuda.stream(s_d2h):
+                ho[l]["idx"].copy_(sl["idx"][:tot], non_blocking=True)
+                ho[l]["cu"].copy_(sl["cu"], non_blocking=True)
+                ho[l]["ko"].copy_(sl["ko"][:tot], non_blocking=True)
+                ho[l]["vo"].copy_(sl["vo"][:tot], non_blocking=True)
+                d2h_done[s].record(s_d2h)
+
+    step()
+    torch.cuda.synchronize(dev)
+    K = args.e2e_steps
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    for _ in range(K):
+        step()
+    torch.cuda.synchronize(dev)
+    dt = (time.perf_counter() - t0) / K
+    barrier(world)
+    dt = max_over_ranks(dt, world)
+    for sl in slots:
+        st = sg.sgdkv_last_error(sl["ws"])
+        if st != sg.OK:
+            raise RuntimeError(f"device-side error in the e2e run: {sg.status_string(st)}")
+    return {"value": world * wl.L * Ls / dt, "unit": UNIT, "h2d_bytes_per_step": int(h2d_bytes),
+            "d2h_bytes_per_step": int(d2h_bytes), "ms_per_step": dt * 1e3, "steps": K,
+            "overlap": "H2D / compute / D2H on three streams, two device slots"}
+
+
+# ------------------------------------------------------------------------------------------
+# the CPU oracle (reported baseline; also the reference arm)
+# ------------------------------------------------------------------------------------------
+
+def cpu_child(args):
+    """Runs in a fresh process: times the oracle on one layer (all KV heads) of the workload."""
+    import numpy as np
+
+    from oracle import sgdkv_oracle as O
+    from paper_2609_03235_gb300 import configs, synth
+    wl = configs.BY_NAME[args.workload]
+    heads = int(os.environ.get("SGDKV_ORACLE_HEADS", str(wl.Hkv)))
+    inp = synth.layer_inputs_host(wl, 0)
+    n_sink, n_recent = configs.sink_recent_split(wl.floor)
+    b_all = O.allocate_budgets(synth.head_scores(wl), wl.L, wl.total_budget(args.frac), wl.floor)
+    b = b_all[:wl.Hkv][:heads]
+    G = wl.G
+    reps = int(os.environ.get("SGDKV_ORACLE_REPS", "1"))
+    times = []
+    for _ in range(reps):
+        t0 = time.perf_counter()
+        O.allocate_budgets(synth.head_scores(wl), wl.L, wl.total_budget(args.frac), wl.floor)
+        O.compress_layer(inp["q"][:heads * G], inp["K"][:heads], inp["V"][:heads], b, n_sink,
+                         n_recent, pool=wl.pool)
+        times.append(time.perf_counter() - t0)
+    print(json.dumps({"seconds": times, "heads": heads, "Hkv": wl.Hkv,
+                      "threads": int(os.environ.get("OMP_NUM_THREADS", "0"))}))
+
+
+def run_cpu_oracle(args, heads=None, reps=1):
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    env = dict(os.environ)
+    for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        env[v] = str(cores)
+    env["CUDA_VISIBLE_DEVICES"] = ""
+    if heads is not None:
+        env["SGDKV_ORACLE_HEADS"] = str(heads)
+    env["SGDKV_ORACLE_REPS"] = str(reps)
+    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--cpu-child", "--workload",
+           args.workload, "--frac", str(args.frac)]
+    r = subprocess.run(cmd, env=env, capture_output=True, text=True, timeout=1800)
+    if r.returncode != 0:
+        raise RuntimeError("oracle child failed:\n" + r.stderr[-2000:])
+    out = json.loads(r.stdout.strip().splitlines()[-1])
+    return out, cores
+
+
+def cpu_baseline(args):
+    from paper_2609_03235_gb300 import configs
+    wl = configs.BY_NAME[args.workload]
+    out, cores = run_cpu_oracle(args, reps=3)
+    sec = statistics.mean(out["seconds"])
+    per_layer = sec * wl.Hkv / out["heads"]
+    return {"value": wl.L / per_layer, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"1 of {wl.n_layers} layers ({out['heads']} of {wl.Hkv} KV heads), "
+                      f"mean of 3 runs, {sec:.1f} s each, NumPy float64 oracle, BLAS threads = {cores}"}
+
+
+def run_reference(args, world, rank):
+    from paper_2609_03235_gb300 import configs
+    wl = configs.BY_NAME[args.workload]
+    if rank != 0:
+        return None
+    # each step: one KV head of one layer (a bounded sample of the workload)
+    out, cores = run_cpu_oracle(args, heads=1, reps=args.warmup + args.steps)
+    secs = out["seconds"][args.warmup:] or out["seconds"]
+    step_s = statistics.mean(secs)
+    value = wl.L / (step_s * wl.Hkv)
+    return {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded, host-generated)", "impl": "reference",
+            "config": {"workload": wl.name, "budget_frac": args.frac},
+            "cpu_baseline": {"value": value, "unit": UNIT, "kind": "oracle", "cores": cores,
+                             "sample": f"each step: 1 KV head of 1 layer of {wl.name}"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    if args.cpu_child:
+        cpu_child(args)
+        return 0
+    world, rank, local = dist_env()
+    if args.gpus != world and world > 1:
+        print(f"warning: --gpus {args.gpus} but WORLD_SIZE {world}", file=sys.stderr)
+    if args.impl == "reference":
+        rec = run_reference(args, world, rank)
+        if rec is not None:
+            print(json.dumps(rec))
+        return 0
+    dist_init(world)
+    rec = run_ours(args, world, rank, local)
+    if rank == 0:
+        if world == 1 and not args.no_cpu_baseline:
+            rec["cpu_baseline"] = cpu_baseline(args)
+        print(json.dumps(rec))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

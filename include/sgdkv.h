@@ -1,0 +1,170 @@
+/*
+ * sgdkv.h: C-ABI of libsgdkv, the GB300 (sm_103a) implementation of the SGD-KV
+ * inference-time KV-cache compression step ("Summarization Guided KV Cache Compression").
+ *
+ * Per layer, after prefill, the step
+ *   1. scores every cached token of each KV head with the last W window queries
+ *      (causal softmax of q.k/sqrt(d), summed over the window and the GQA group),
+ *   2. smooths the scores with a 1-D max-pool,
+ *   3. keeps each head's b_h best tokens (sink and recent tokens always kept), where b_h
+ *      comes from the summarization-score budget allocation of Section 3.3 / Algorithm 1,
+ *   4. gathers the kept K/V rows into a flat per-head variable-length cache.
+ *
+ * Conventions shared by every entry point:
+ *   - The caller owns all memory.  The library allocates nothing and keeps no pointer past
+ *     a call.  Device buffers are plain device pointers (cudaMalloc or torch storage).
+ *   - bf16 tensors are passed as `const void*` to raw bfloat16 storage, row-major:
+ *       q_win [Hq][W][d]     window queries, query head q belongs to KV head q / (Hq/Hkv)
+ *       K, V  [Hkv][L][d]    one layer's prefilled cache
+ *     Every device pointer must be 16-byte aligned.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).  Device
+ *     work is enqueued asynchronously on it; host-side argument checks happen before any
+ *     launch and leave all outputs untouched on error.
+ *   - `workspace` is a device buffer of at least sgdkv_workspace_bytes(...) bytes, 256-byte
+ *     aligned, zero-filled once by the caller before its first use.  The library keeps it
+ *     in a reusable state after every call.  Calls that share a workspace must be ordered
+ *     (same stream or synchronised); calls with separate workspaces may run concurrently.
+ *   - Device-side failures (a bounded wait that ran out) are recorded in a status word in
+ *     the workspace and reported by sgdkv_last_error.  No call aborts the process, traps,
+ *     or falls back to the CPU.
+ *   - v1 limits: d == 128; Hq % Hkv == 0; G*W a multiple of 32 and <= 512 (G = Hq/Hkv);
+ *     Hkv <= SGDKV_MAX_KV_HEADS; Hkv*L < 2^31; pool odd in [1, 63].
+ */
+#ifndef SGDKV_H_
+#define SGDKV_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SGDKV_API __attribute__((visibility("default")))
+#else
+#define SGDKV_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SGDKV_MAX_KV_HEADS 64
+#define SGDKV_HEAD_DIM 128
+
+typedef enum {
+  SGDKV_OK = 0,
+  SGDKV_ERR_INVALID_ARG = 1,       /* null pointer, bad shape, misaligned pointer        */
+  SGDKV_ERR_INFEASIBLE_BUDGET = 2, /* total budget outside [N*floor, N*context_len]      */
+  SGDKV_ERR_WORKSPACE = 3,         /* workspace missing, too small or misaligned         */
+  SGDKV_ERR_CUDA = 4,              /* a CUDA runtime call or launch failed               */
+  SGDKV_ERR_TIMEOUT = 5,           /* a device-side bounded wait ran out                 */
+  SGDKV_ERR_UNSUPPORTED = 6,       /* shape outside the v1 limits above                  */
+  SGDKV_ERR_INTERNAL = 7           /* a device-side consistency check failed; the access */
+                                   /* it guarded was skipped                             */
+} sgdkv_status;
+
+/* Allocation modes of sgdkv_allocate_budgets. */
+#define SGDKV_ALLOC_GREEDY 0       /* Algorithm 1, excess to top-scoring heads in turn     */
+#define SGDKV_ALLOC_PROPORTIONAL 1 /* water level: min(cap, lambda * S_h)                  */
+#define SGDKV_ALLOC_THRESHOLD 2    /* appendix "thr": scores below the mean zeroed, greedy */
+
+/* Static description of a status code. Never NULL. */
+SGDKV_API const char* sgdkv_status_string(int status);
+
+/* Library version, major*10000 + minor*100 + patch. */
+SGDKV_API int sgdkv_version(void);
+
+/*
+ * Head-level budget allocation (host only, deterministic, no device work).
+ * Follows Section 3.3, Eq. (2) and Appendix A.1, Algorithm 1 of the paper.
+ *
+ * head_scores  [n_heads] host floats, one summarization score per (layer, KV head); the
+ *              allocation runs jointly over all of them.  Finite, >= 0; all zero means
+ *              uniform.
+ * context_len  C, tokens per head before compression.
+ * total_budget T, kept tokens summed over all heads, floors included.
+ * floor        f = b_sink + b_window, kept by every head; the middle share is capped at
+ *              M = C - f.
+ * mode         SGDKV_ALLOC_*.
+ * budgets_out  [n_heads] host int64: f <= b_h <= C and sum b_h == T exactly.
+ *
+ * The middle pool P = T - n_heads*f is shared in proportion to S_h = s_h / sum(s)
+ * (Eq. 2), shares above M are capped and their excess redistributed (Algorithm 1), and
+ * the real shares are rounded by largest remainder (ties: higher S_h, then lower index).
+ * All arithmetic is IEEE double in a fixed order, so results are bit-reproducible.
+ * Errors: INVALID_ARG (null, n_heads <= 0, f outside [0, C], bad mode, negative/NaN/Inf
+ * score), INFEASIBLE_BUDGET (T outside [n*f, n*C]).  budgets_out untouched on error.
+ */
+SGDKV_API sgdkv_status sgdkv_allocate_budgets(const float* head_scores, int32_t n_heads,
+                                    int64_t context_len, int64_t total_budget, int64_t floor,
+                                    int32_t mode, int64_t* budgets_out);
+
+/* Workspace bytes needed by sgdkv_score / sgdkv_compact / sgdkv_compress_layer for this
+ * shape (one size serves all three).  Returns 0 for shapes outside the v1 limits. */
+SGDKV_API size_t sgdkv_workspace_bytes(int32_t Hq, int32_t Hkv, int64_t L, int32_t d, int32_t W);
+
+/*
+ * Window scoring (Section 3.3 and Section 5: cumulative attention of the final
+ * observation window, SnapKV-style), followed by max-pooling.
+ *
+ *   raw[h][j]    = sum_{g<G} sum_{w<W} softmax_j( q[h*G+g][w] . K[h][j] / sqrt(d) )
+ *                  where window query w sits at position L-W+w and sees keys j <= L-W+w;
+ *   scores[h][j] = max of raw[h][t] over t in [j - pool/2, j + pool/2] within [0, L).
+ *
+ * q_win      device bf16 [Hq][W][d];  K  device bf16 [Hkv][L][d]
+ * pool       odd kernel size; 1 returns the raw scores.
+ * scores_out device fp32 [Hkv][L].
+ * Errors: INVALID_ARG, UNSUPPORTED, WORKSPACE, CUDA (launch failure).
+ */
+SGDKV_API sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq, int32_t Hkv, int64_t L,
+                         int32_t d, int32_t W, int32_t pool, float* scores_out,
+                         void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * Token selection and gather (Section 3.3): per KV head keep positions [0, n_sink) and
+ * [L - n_recent, L), plus the (b_h - n_sink - n_recent) middle positions with the highest
+ * scores (equal scores: lower position first).  Kept positions are written ascending.
+ *
+ * K, V            device bf16 [Hkv][L][d]
+ * scores          device fp32 [Hkv][L], finite and >= 0 (as produced by sgdkv_score)
+ * budgets         HOST int64 [Hkv], n_sink + n_recent <= b_h <= L
+ * indices_out     device int32 [sum b_h]: kept positions, head by head
+ * cu_seqlens_out  device int32 [Hkv + 1]: cu[0] = 0, cu[h+1] = cu[h] + b_h
+ * K_out, V_out    device bf16 [sum b_h][d]: row cu[h]+i = K[h][indices_out[cu[h]+i]]
+ * Errors: INVALID_ARG, UNSUPPORTED, WORKSPACE, CUDA.
+ */
+SGDKV_API sgdkv_status sgdkv_compact(const void* K, const void* V, const float* scores,
+                           const int64_t* budgets, int32_t Hkv, int64_t L, int32_t d,
+                           int64_t n_sink, int64_t n_recent, int32_t* indices_out,
+                           int32_t* cu_seqlens_out, void* K_out, void* V_out, void* workspace,
+                           size_t ws_bytes, void* stream);
+
+/*
+ * The whole per-layer step: sgdkv_score followed by sgdkv_compact on the same stream,
+ * keeping the pooled scores in the workspace.  scores_out may be NULL; when given, it
+ * receives the pooled scores as sgdkv_score would.  Other arguments as above.
+ */
+SGDKV_API sgdkv_status sgdkv_compress_layer(const void* q_win, const void* K, const void* V,
+                                  const int64_t* budgets, int32_t Hq, int32_t Hkv, int64_t L,
+                                  int32_t d, int32_t W, int32_t pool, int64_t n_sink,
+                                  int64_t n_recent, float* scores_out, int32_t* indices_out,
+                                  int32_t* cu_seqlens_out, void* K_out, void* V_out,
+                                  void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * Diagnostics: number of kernel launches this process has issued through libsgdkv so far
+ * (all entry points, all devices).  No counterpart in the paper; used to report how many
+ * of the library's kernels a timed region ran.
+ */
+SGDKV_API uint64_t sgdkv_launch_count(void);
+
+/*
+ * Synchronises `stream`, then returns and clears the first device-side failure recorded
+ * in `workspace` since the last call (SGDKV_OK if none), or SGDKV_ERR_CUDA if the stream
+ * itself reports an error.
+ */
+SGDKV_API sgdkv_status sgdkv_last_error(void* workspace, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SGDKV_H_ */

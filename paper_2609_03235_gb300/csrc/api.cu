@@ -1,0 +1,227 @@
+// C-ABI entry points of libsgdkv: argument checks, workspace carving, launches.
+#include <atomic>
+#include <cstdint>
+#include <cstring>
+
+#include "sgdkv_internal.cuh"
+
+namespace sgdkv {
+
+namespace {
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+}  // namespace
+
+namespace {
+std::atomic<uint64_t> g_launches{0};
+}  // namespace
+
+void note_launches(int n) { g_launches.fetch_add(uint64_t(n), std::memory_order_relaxed); }
+
+WsLayout workspace_layout(int32_t Hkv, int64_t L) {
+  WsLayout w{};
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align256(off + bytes);
+    return at;
+  };
+  const size_t H = size_t(Hkv);
+  const size_t n_sel_chunks = size_t(ceil_div(L, kSelChunk));
+  w.status = take(256);
+  w.merge_cnt = take(H * sizeof(uint32_t));
+  w.sel = take(H * sizeof(SelState));
+  w.hist = take(H * 256 * sizeof(uint32_t));
+  w.sel_cnt = take(H * sizeof(uint32_t));
+  w.chunk_cnt = take(H * n_sel_chunks * sizeof(uint2));
+  w.lse = take(H * kMaxRows * sizeof(float));
+  w.partial = take(H * size_t(kMaxScoreParts) * kMaxRows * sizeof(float2));
+  w.raw = take(H * size_t(L) * sizeof(float));
+  w.pooled = take(H * size_t(L) * sizeof(float));
+  w.total = off;
+  return w;
+}
+
+Ws workspace_view(void* base, const WsLayout& lay) {
+  char* b = static_cast<char*>(base);
+  Ws ws;
+  ws.status = reinterpret_cast<uint32_t*>(b + lay.status);
+  ws.merge_cnt = reinterpret_cast<uint32_t*>(b + lay.merge_cnt);
+  ws.sel = reinterpret_cast<SelState*>(b + lay.sel);
+  ws.hist = reinterpret_cast<uint32_t*>(b + lay.hist);
+  ws.sel_cnt = reinterpret_cast<uint32_t*>(b + lay.sel_cnt);
+  ws.chunk_cnt = reinterpret_cast<uint2*>(b + lay.chunk_cnt);
+  ws.lse = reinterpret_cast<float*>(b + lay.lse);
+  ws.partial = reinterpret_cast<float2*>(b + lay.partial);
+  ws.raw = reinterpret_cast<float*>(b + lay.raw);
+  ws.pooled = reinterpret_cast<float*>(b + lay.pooled);
+  return ws;
+}
+
+namespace {
+
+// Shape limits of v1 (see sgdkv.h).  Returns SGDKV_OK or the error to report.
+sgdkv_status check_score_shape(int32_t Hq, int32_t Hkv, int64_t L, int32_t d, int32_t W) {
+  if (Hq <= 0 || Hkv <= 0 || L <= 0 || d <= 0 || W <= 0) return SGDKV_ERR_INVALID_ARG;
+  if (Hq % Hkv != 0 || W > L) return SGDKV_ERR_INVALID_ARG;
+  if (d != kD || Hkv > SGDKV_MAX_KV_HEADS) return SGDKV_ERR_UNSUPPORTED;
+  const int64_t GW = int64_t(Hq / Hkv) * W;
+  if (GW > kMaxRows || GW % 32 != 0) return SGDKV_ERR_UNSUPPORTED;
+  if (int64_t(Hkv) * L >= (int64_t(1) << 31)) return SGDKV_ERR_UNSUPPORTED;
+  return SGDKV_OK;
+}
+
+sgdkv_status check_workspace(void* ws, size_t ws_bytes, int32_t Hkv, int64_t L) {
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return SGDKV_ERR_WORKSPACE;
+  if (ws_bytes < workspace_layout(Hkv, L).total) return SGDKV_ERR_WORKSPACE;
+  return SGDKV_OK;
+}
+
+sgdkv_status check_pool(int32_t pool) {
+  if (pool < 1 || pool > 63 || pool % 2 == 0) return SGDKV_ERR_INVALID_ARG;
+  return SGDKV_OK;
+}
+
+// Validates budgets and fills the per-head table; returns the total kept rows.
+sgdkv_status build_head_table(const int64_t* budgets, int32_t Hkv, int64_t L, int64_t n_sink,
+                              int64_t n_recent, HeadTable* ht, int64_t* total) {
+  if (!budgets) return SGDKV_ERR_INVALID_ARG;
+  if (n_sink < 0 || n_recent < 0 || n_sink + n_recent > L) return SGDKV_ERR_INVALID_ARG;
+  std::memset(ht, 0, sizeof(*ht));
+  ht->Hkv = Hkv;
+  ht->L = L;
+  ht->n_sink = n_sink;
+  ht->n_recent = n_recent;
+  int64_t acc = 0;
+  ht->cu[0] = 0;
+  for (int h = 0; h < Hkv; ++h) {
+    const int64_t b = budgets[h];
+    if (b < n_sink + n_recent || b > L) return SGDKV_ERR_INVALID_ARG;
+    ht->k_mid[h] = int32_t(b - n_sink - n_recent);
+    acc += b;
+    ht->cu[h + 1] = int32_t(acc);
+  }
+  *total = acc;
+  return SGDKV_OK;
+}
+
+sgdkv_status from_cuda(cudaError_t e) { return e == cudaSuccess ? SGDKV_OK : SGDKV_ERR_CUDA; }
+
+}  // namespace
+}  // namespace sgdkv
+
+using namespace sgdkv;
+
+extern "C" {
+
+const char* sgdkv_status_string(int status) {
+  switch (status) {
+    case SGDKV_OK: return "ok";
+    case SGDKV_ERR_INVALID_ARG: return "invalid argument";
+    case SGDKV_ERR_INFEASIBLE_BUDGET: return "infeasible budget";
+    case SGDKV_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
+    case SGDKV_ERR_CUDA: return "CUDA error";
+    case SGDKV_ERR_TIMEOUT: return "device-side wait timed out";
+    case SGDKV_ERR_UNSUPPORTED: return "shape outside the supported limits";
+    case SGDKV_ERR_INTERNAL: return "device-side consistency check failed";
+    default: return "unknown status";
+  }
+}
+
+int sgdkv_version(void) { return 100; }
+
+uint64_t sgdkv_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+size_t sgdkv_workspace_bytes(int32_t Hq, int32_t Hkv, int64_t L, int32_t d, int32_t W) {
+  if (check_score_shape(Hq, Hkv, L, d, W) != SGDKV_OK) return 0;
+  return workspace_layout(Hkv, L).total;
+}
+
+sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq, int32_t Hkv, int64_t L,
+                         int32_t d, int32_t W, int32_t pool, float* scores_out,
+                         void* workspace, size_t ws_bytes, void* stream) {
+  if (!q_win || !K || !scores_out) return SGDKV_ERR_INVALID_ARG;
+  if (!aligned16(q_win) || !aligned16(K) || !aligned16(scores_out)) return SGDKV_ERR_INVALID_ARG;
+  sgdkv_status s = check_score_shape(Hq, Hkv, L, d, W);
+  if (s != SGDKV_OK) return s;
+  if ((s = check_pool(pool)) != SGDKV_OK) return s;
+  if ((s = check_workspace(workspace, ws_bytes, Hkv, L)) != SGDKV_OK) return s;
+  const Ws ws = workspace_view(workspace, workspace_layout(Hkv, L));
+  return from_cuda(launch_score(static_cast<const __nv_bfloat16*>(q_win),
+                                static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, pool,
+                                scores_out, ws, static_cast<cudaStream_t>(stream)));
+}
+
+sgdkv_status sgdkv_compact(const void* K, const void* V, const float* scores,
+                           const int64_t* budgets, int32_t Hkv, int64_t L, int32_t d,
+                           int64_t n_sink, int64_t n_recent, int32_t* indices_out,
+                           int32_t* cu_seqlens_out, void* K_out, void* V_out, void* workspace,
+                           size_t ws_bytes, void* stream) {
+  if (!K || !V || !scores || !cu_seqlens_out) return SGDKV_ERR_INVALID_ARG;
+  if (Hkv <= 0 || L <= 0 || d <= 0) return SGDKV_ERR_INVALID_ARG;
+  if (d != kD || Hkv > SGDKV_MAX_KV_HEADS || int64_t(Hkv) * L >= (int64_t(1) << 31))
+    return SGDKV_ERR_UNSUPPORTED;
+  if (!aligned16(K) || !aligned16(V) || !aligned16(scores)) return SGDKV_ERR_INVALID_ARG;
+  HeadTable ht;
+  int64_t total = 0;
+  sgdkv_status s = build_head_table(budgets, Hkv, L, n_sink, n_recent, &ht, &total);
+  if (s != SGDKV_OK) return s;
+  if (total > 0 && (!indices_out || !K_out || !V_out)) return SGDKV_ERR_INVALID_ARG;
+  if (total > 0 && (!aligned16(K_out) || !aligned16(V_out))) return SGDKV_ERR_INVALID_ARG;
+  if ((s = check_workspace(workspace, ws_bytes, Hkv, L)) != SGDKV_OK) return s;
+  const Ws ws = workspace_view(workspace, workspace_layout(Hkv, L));
+  return from_cuda(launch_compact(static_cast<const __nv_bfloat16*>(K),
+                                  static_cast<const __nv_bfloat16*>(V), scores, ht, indices_out,
+                                  cu_seqlens_out, static_cast<__nv_bfloat16*>(K_out),
+                                  static_cast<__nv_bfloat16*>(V_out), total, ws,
+                                  static_cast<cudaStream_t>(stream)));
+}
+
+sgdkv_status sgdkv_compress_layer(const void* q_win, const void* K, const void* V,
+                                  const int64_t* budgets, int32_t Hq, int32_t Hkv, int64_t L,
+                                  int32_t d, int32_t W, int32_t pool, int64_t n_sink,
+                                  int64_t n_recent, float* scores_out, int32_t* indices_out,
+                                  int32_t* cu_seqlens_out, void* K_out, void* V_out,
+                                  void* workspace, size_t ws_bytes, void* stream) {
+  if (!q_win || !K || !V || !cu_seqlens_out) return SGDKV_ERR_INVALID_ARG;
+  if (!aligned16(q_win) || !aligned16(K) || !aligned16(V)) return SGDKV_ERR_INVALID_ARG;
+  if (scores_out && !aligned16(scores_out)) return SGDKV_ERR_INVALID_ARG;
+  sgdkv_status s = check_score_shape(Hq, Hkv, L, d, W);
+  if (s != SGDKV_OK) return s;
+  if ((s = check_pool(pool)) != SGDKV_OK) return s;
+  HeadTable ht;
+  int64_t total = 0;
+  if ((s = build_head_table(budgets, Hkv, L, n_sink, n_recent, &ht, &total)) != SGDKV_OK) return s;
+  if (total > 0 && (!indices_out || !K_out || !V_out)) return SGDKV_ERR_INVALID_ARG;
+  if (total > 0 && (!aligned16(K_out) || !aligned16(V_out))) return SGDKV_ERR_INVALID_ARG;
+  if ((s = check_workspace(workspace, ws_bytes, Hkv, L)) != SGDKV_OK) return s;
+  const Ws ws = workspace_view(workspace, workspace_layout(Hkv, L));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  float* pooled = scores_out ? scores_out : ws.pooled;
+  cudaError_t e = launch_score(static_cast<const __nv_bfloat16*>(q_win),
+                               static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, pool,
+                               pooled, ws, st);
+  if (e != cudaSuccess) return SGDKV_ERR_CUDA;
+  return from_cuda(launch_compact(static_cast<const __nv_bfloat16*>(K),
+                                  static_cast<const __nv_bfloat16*>(V), pooled, ht, indices_out,
+                                  cu_seqlens_out, static_cast<__nv_bfloat16*>(K_out),
+                                  static_cast<__nv_bfloat16*>(V_out), total, ws, st));
+}
+
+sgdkv_status sgdkv_last_error(void* workspace, void* stream) {
+  if (!workspace) return SGDKV_ERR_WORKSPACE;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint32_t code = 0;
+  if (cudaMemcpyAsync(&code, workspace, sizeof(code), cudaMemcpyDeviceToHost, st) != cudaSuccess)
+    return SGDKV_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return SGDKV_ERR_CUDA;
+  if (code != 0) {
+    const uint32_t zero = 0;
+    if (cudaMemcpyAsync(workspace, &zero, sizeof(zero), cudaMemcpyHostToDevice, st) != cudaSuccess)
+      return SGDKV_ERR_CUDA;
+    if (cudaStreamSynchronize(st) != cudaSuccess) return SGDKV_ERR_CUDA;
+  }
+  return static_cast<sgdkv_status>(code);
+}
+
+}  // extern "C"

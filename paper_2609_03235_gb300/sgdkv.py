@@ -1,0 +1,177 @@
+"""Thin Python binding of libsgdkv (include/sgdkv.h), same names as the C-ABI.
+
+Argument marshalling only: every step of the compression path runs in the CUDA library.
+Tensors are torch tensors (device memory, caller-owned); host arrays are NumPy.  If the
+library has not been built, every call raises ``LibraryMissing``; there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "lib", "libsgdkv.so")
+
+OK, ERR_INVALID_ARG, ERR_INFEASIBLE_BUDGET, ERR_WORKSPACE, ERR_CUDA, ERR_TIMEOUT, \
+    ERR_UNSUPPORTED, ERR_INTERNAL = range(8)
+ALLOC_GREEDY, ALLOC_PROPORTIONAL, ALLOC_THRESHOLD = 0, 1, 2
+EXPORTED = ("sgdkv_status_string", "sgdkv_version", "sgdkv_allocate_budgets",
+            "sgdkv_workspace_bytes", "sgdkv_score", "sgdkv_compact", "sgdkv_compress_layer",
+            "sgdkv_last_error", "sgdkv_launch_count")
+
+
+class LibraryMissing(RuntimeError):
+    pass
+
+
+class SgdkvError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} (status {status})")
+
+
+_lib = None
+_P = ctypes.c_void_p
+_I32, _I64, _SZ = ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+
+
+def lib():
+    """The loaded libsgdkv.so (loaded once)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise LibraryMissing(f"{LIB_PATH} not built: run `python -c \"import __graft_entry__ as g; g.build()\"`")
+        L = ctypes.CDLL(LIB_PATH)
+        L.sgdkv_status_string.restype = ctypes.c_char_p
+        L.sgdkv_status_string.argtypes = [ctypes.c_int]
+        L.sgdkv_version.restype = ctypes.c_int
+        L.sgdkv_allocate_budgets.restype = ctypes.c_int
+        L.sgdkv_allocate_budgets.argtypes = [_P, _I32, _I64, _I64, _I64, _I32, _P]
+        L.sgdkv_workspace_bytes.restype = _SZ
+        L.sgdkv_workspace_bytes.argtypes = [_I32, _I32, _I64, _I32, _I32]
+        L.sgdkv_score.restype = ctypes.c_int
+        L.sgdkv_score.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, _I32, _P, _P, _SZ, _P]
+        L.sgdkv_compact.restype = ctypes.c_int
+        L.sgdkv_compact.argtypes = [_P, _P, _P, _P, _I32, _I64, _I32, _I64, _I64, _P, _P, _P, _P,
+                                    _P, _SZ, _P]
+        L.sgdkv_compress_layer.restype = ctypes.c_int
+        L.sgdkv_compress_layer.argtypes = [_P, _P, _P, _P, _I32, _I32, _I64, _I32, _I32, _I32,
+                                           _I64, _I64, _P, _P, _P, _P, _P, _P, _SZ, _P]
+        L.sgdkv_last_error.restype = ctypes.c_int
+        L.sgdkv_last_error.argtypes = [_P, _P]
+        L.sgdkv_launch_count.restype = ctypes.c_uint64
+        _lib = L
+    return _lib
+
+
+def status_string(status: int) -> str:
+    return lib().sgdkv_status_string(int(status)).decode()
+
+
+def _check(status: int, where: str):
+    if status != OK:
+        raise SgdkvError(status, where)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(int(getattr(stream, "cuda_stream", stream)))
+
+
+def sgdkv_version() -> int:
+    return lib().sgdkv_version()
+
+
+def sgdkv_allocate_budgets(head_scores, context_len: int, total_budget: int, floor: int,
+                           mode: int = ALLOC_GREEDY) -> np.ndarray:
+    s = np.ascontiguousarray(head_scores, dtype=np.float32)
+    out = np.zeros(s.size, dtype=np.int64)
+    st = lib().sgdkv_allocate_budgets(s.ctypes.data_as(_P), s.size, int(context_len),
+                                      int(total_budget), int(floor), int(mode),
+                                      out.ctypes.data_as(_P))
+    _check(st, "sgdkv_allocate_budgets")
+    return out
+
+
+def sgdkv_workspace_bytes(Hq: int, Hkv: int, L: int, d: int, W: int) -> int:
+    return int(lib().sgdkv_workspace_bytes(Hq, Hkv, L, d, W))
+
+
+def make_workspace(Hq: int, Hkv: int, L: int, W: int, device="cuda", d: int = 128):
+    """Zero-filled workspace tensor for this shape (caller-owned device memory)."""
+    import torch
+    n = sgdkv_workspace_bytes(Hq, Hkv, L, d, W)
+    if n == 0:
+        raise SgdkvError(ERR_UNSUPPORTED, "sgdkv_workspace_bytes")
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def sgdkv_score(q_win, K, W: int, pool: int, scores_out, workspace, stream=None):
+    Hq, W_, d = q_win.shape
+    Hkv, L, _ = K.shape
+    st = lib().sgdkv_score(_ptr(q_win), _ptr(K), Hq, Hkv, L, d, W, pool, _ptr(scores_out),
+                           _ptr(workspace), workspace.numel(), _stream(stream))
+    _check(st, "sgdkv_score")
+
+
+def _budgets(b):
+    return np.ascontiguousarray(b, dtype=np.int64)
+
+
+def sgdkv_compact(K, V, scores, budgets, n_sink: int, n_recent: int, indices_out,
+                  cu_seqlens_out, K_out, V_out, workspace, stream=None):
+    Hkv, L, d = K.shape
+    b = _budgets(budgets)
+    st = lib().sgdkv_compact(_ptr(K), _ptr(V), _ptr(scores), b.ctypes.data_as(_P), Hkv, L, d,
+                             n_sink, n_recent, _ptr(indices_out), _ptr(cu_seqlens_out),
+                             _ptr(K_out), _ptr(V_out), _ptr(workspace), workspace.numel(),
+                             _stream(stream))
+    _check(st, "sgdkv_compact")
+
+
+def sgdkv_compress_layer(q_win, K, V, budgets, W: int, pool: int, n_sink: int, n_recent: int,
+                         scores_out, indices_out, cu_seqlens_out, K_out, V_out, workspace,
+                         stream=None):
+    Hq, _, d = q_win.shape
+    Hkv, L, _ = K.shape
+    b = _budgets(budgets)
+    st = lib().sgdkv_compress_layer(_ptr(q_win), _ptr(K), _ptr(V), b.ctypes.data_as(_P), Hq,
+                                    Hkv, L, d, W, pool, n_sink, n_recent, _ptr(scores_out),
+                                    _ptr(indices_out), _ptr(cu_seqlens_out), _ptr(K_out),
+                                    _ptr(V_out), _ptr(workspace), workspace.numel(),
+                                    _stream(stream))
+    _check(st, "sgdkv_compress_layer")
+
+
+def sgdkv_launch_count() -> int:
+    return int(lib().sgdkv_launch_count())
+
+
+def sgdkv_last_error(workspace, stream=None) -> int:
+    return int(lib().sgdkv_last_error(_ptr(workspace), _stream(stream)))
+
+
+def compress_layer_alloc(q_win, K, V, budgets, W: int, pool: int, n_sink: int, n_recent: int,
+                         workspace, stream=None, want_scores: bool = True):
+    """Allocates the outputs with torch, calls sgdkv_compress_layer, returns them."""
+    import torch
+    Hkv, L, d = K.shape
+    total = int(np.sum(_budgets(budgets)))
+    dev = K.device
+    scores = torch.empty((Hkv, L), dtype=torch.float32, device=dev) if want_scores else None
+    idx = torch.empty(max(total, 1), dtype=torch.int32, device=dev)
+    cu = torch.empty(Hkv + 1, dtype=torch.int32, device=dev)
+    ko = torch.empty((max(total, 1), d), dtype=K.dtype, device=dev)
+    vo = torch.empty((max(total, 1), d), dtype=V.dtype, device=dev)
+    sgdkv_compress_layer(q_win, K, V, budgets, W, pool, n_sink, n_recent, scores, idx, cu, ko,
+                         vo, workspace, stream)
+    return dict(scores=scores, indices=idx[:total], cu_seqlens=cu, K_out=ko[:total],
+                V_out=vo[:total])

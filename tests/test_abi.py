@@ -1,0 +1,136 @@
+"""Host-side checks of libsgdkv (no GPU needed): the library loads, exports every entry
+point declared in include/sgdkv.h, its host allocator equals the oracle bit for bit, and
+argument checks reject bad calls before any device work."""
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import sgdkv_oracle as O
+from paper_2609_03235_gb300 import sgdkv as sg
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built_library():
+    if not os.path.exists(sg.LIB_PATH):
+        from paper_2609_03235_gb300 import build_lib
+        build_lib.build()
+    return sg.lib()
+
+
+def _declared_symbols():
+    text = open(os.path.join(ROOT, "include", "sgdkv.h")).read()
+    return sorted(set(re.findall(r"SGDKV_API[^;]*?\b(sgdkv_\w+)\s*\(", text, re.S)))
+
+
+def test_exports_every_declared_symbol():
+    import ctypes
+    declared = _declared_symbols()
+    assert set(declared) == set(sg.EXPORTED)
+    handle = ctypes.CDLL(sg.LIB_PATH)
+    for name in declared:
+        assert hasattr(handle, name), name
+
+
+def test_status_strings_and_version():
+    assert sg.status_string(sg.OK) == "ok"
+    assert "timed out" in sg.status_string(sg.ERR_TIMEOUT)
+    assert sg.status_string(999) == "unknown status"
+    assert sg.sgdkv_version() >= 100
+
+
+def _random_alloc_case(rng):
+    n = int(rng.integers(1, 700))
+    dist = rng.integers(0, 3)
+    if dist == 0:
+        s = rng.beta(0.5, 2.0, n)
+    elif dist == 1:
+        s = rng.random(n)
+    else:
+        s = rng.integers(0, 3, n) * 0.5        # many exact ties, some zeros
+    s = s.astype(np.float32)
+    C = int(rng.integers(16, 1 << 21))
+    f = int(rng.integers(0, C // 2 + 1))
+    T = int(rng.integers(n * f, n * C + 1))
+    return s, C, T, f
+
+
+@pytest.mark.parametrize("mode", [sg.ALLOC_GREEDY, sg.ALLOC_PROPORTIONAL, sg.ALLOC_THRESHOLD])
+def test_allocator_bit_exact_vs_oracle(mode):
+    rng = np.random.default_rng(2024 + mode)
+    for _ in range(150):
+        s, C, T, f = _random_alloc_case(rng)
+        got = sg.sgdkv_allocate_budgets(s, C, T, f, mode)
+        exp = O.allocate_budgets(s, C, T, f, mode)
+        assert np.array_equal(got, exp), (s[:8], C, T, f, mode)
+
+
+def test_allocator_on_workload_head_scores():
+    from paper_2609_03235_gb300 import configs, synth
+    for wl in configs.WORKLOADS:
+        s = synth.head_scores(wl)
+        for frac in wl.budget_fracs:
+            T = wl.total_budget(frac)
+            got = sg.sgdkv_allocate_budgets(s, wl.L, T, wl.floor)
+            assert np.array_equal(got, O.allocate_budgets(s, wl.L, T, wl.floor))
+            assert got.sum() == T
+
+
+@pytest.mark.parametrize("args,status", [
+    ((np.array([1.0, -1.0], np.float32), 100, 120, 10), sg.ERR_INVALID_ARG),
+    ((np.array([1.0, np.nan], np.float32), 100, 120, 10), sg.ERR_INVALID_ARG),
+    ((np.array([1.0, 1.0], np.float32), 100, 19, 10), sg.ERR_INFEASIBLE_BUDGET),
+    ((np.array([1.0, 1.0], np.float32), 100, 201, 10), sg.ERR_INFEASIBLE_BUDGET),
+    ((np.array([1.0, 1.0], np.float32), 100, 150, 101), sg.ERR_INVALID_ARG),
+])
+def test_allocator_errors(args, status):
+    with pytest.raises(sg.SgdkvError) as e:
+        sg.sgdkv_allocate_budgets(*args)
+    assert e.value.status == status
+
+
+def test_allocator_bad_mode():
+    with pytest.raises(sg.SgdkvError):
+        sg.sgdkv_allocate_budgets(np.ones(3, np.float32), 100, 150, 10, mode=7)
+
+
+def test_workspace_bytes_limits():
+    assert sg.sgdkv_workspace_bytes(28, 4, 131072, 128, 64) > 4 * 131072 * 4
+    assert sg.sgdkv_workspace_bytes(28, 4, 131072, 64, 64) == 0        # d != 128
+    assert sg.sgdkv_workspace_bytes(28, 5, 1000, 128, 32) == 0         # Hq % Hkv != 0
+    assert sg.sgdkv_workspace_bytes(28, 4, 1000, 128, 80) == 0         # G*W > 512
+    assert sg.sgdkv_workspace_bytes(28, 4, 1000, 128, 12) == 0         # G*W % 32 != 0
+    assert sg.sgdkv_workspace_bytes(28, 4, 10, 128, 32) == 0           # W > L
+
+
+def test_score_rejects_bad_args_before_device_work():
+    import ctypes
+    L = sg.lib()
+    buf = (ctypes.c_uint8 * 4096)()
+    p = ctypes.cast(buf, ctypes.c_void_p)
+    # null pointers
+    assert L.sgdkv_score(None, p, 28, 4, 1024, 128, 32, 7, p, p, 4096, None) == sg.ERR_INVALID_ARG
+    # unsupported head dim
+    assert L.sgdkv_score(p, p, 28, 4, 1024, 64, 32, 7, p, p, 1 << 30, None) == sg.ERR_UNSUPPORTED
+    # even pool kernel
+    assert L.sgdkv_score(p, p, 28, 4, 1024, 128, 32, 6, p, p, 1 << 30, None) == sg.ERR_INVALID_ARG
+    # workspace too small
+    assert L.sgdkv_score(p, p, 28, 4, 1024, 128, 32, 7, p, p, 16, None) == sg.ERR_WORKSPACE
+
+
+def test_compact_rejects_bad_budgets():
+    import ctypes
+    L = sg.lib()
+    buf = (ctypes.c_uint8 * 4096)()
+    p = ctypes.cast(buf, ctypes.c_void_p)
+    b = np.array([10, 3], np.int64)   # second head below n_sink + n_recent
+    st = L.sgdkv_compact(p, p, p, b.ctypes.data_as(ctypes.c_void_p), 2, 100, 128, 2, 2, p, p,
+                         p, p, p, 1 << 30, None)
+    assert st == sg.ERR_INVALID_ARG
+    b = np.array([10, 101], np.int64)  # above L
+    st = L.sgdkv_compact(p, p, p, b.ctypes.data_as(ctypes.c_void_p), 2, 100, 128, 2, 2, p, p,
+                         p, p, p, 1 << 30, None)
+    assert st == sg.ERR_INVALID_ARG

@@ -1,0 +1,193 @@
+"""GPU parity of the CUDA path against the CPU oracle, through the C-ABI.
+
+Bars: scores |gpu - oracle| <= 1e-5 + 2e-3 |oracle| element by element; given identical
+scores, indices and cu_seqlens bit-exact; gathered K/V rows bit-exact.  End to end (each
+side with its own scores), the GPU's selection must equal the oracle's selection applied
+to the GPU's scores, and every position where it differs from the oracle's own selection
+must have an oracle score within tolerance of that head's threshold.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import sgdkv_oracle as O
+from paper_2609_03235_gb300 import configs, synth
+from paper_2609_03235_gb300 import sgdkv as sg
+
+pytestmark = pytest.mark.gpu
+RTOL, ATOL = 2e-3, 1e-5
+
+
+@pytest.fixture(scope="module")
+def dev():
+    sg.lib()
+    return torch.device("cuda:0")
+
+
+def _within(got, exp):
+    return np.abs(got.astype(np.float64) - exp) <= ATOL + RTOL * np.abs(exp.astype(np.float64))
+
+
+def _upload(inp, dev):
+    return (synth.to_torch_bf16(inp["q"], dev), synth.to_torch_bf16(inp["K"], dev),
+            synth.to_torch_bf16(inp["V"], dev))
+
+
+SCORE_SHAPES = [
+    # Hq, Hkv, L, W    (G*W = 224, 448, 512, 32, 224 ...)
+    (14, 2, 1000, 32),
+    (28, 4, 3000, 64),
+    (16, 2, 2049, 64),
+    (1, 1, 300, 32),
+    (7, 1, 32, 32),        # L == W: every key is a window key
+    (8, 8, 640, 32),
+    (28, 4, 129, 64),
+]
+
+
+@pytest.mark.parametrize("Hq,Hkv,L,W", SCORE_SHAPES)
+@pytest.mark.parametrize("pool", [1, 7])
+def test_score_parity(dev, Hq, Hkv, L, W, pool):
+    wl = synth.tiny_workload(Hq=Hq, Hkv=Hkv, d=128, L=L, W=W, n_salient=min(8, max(0, L - W - 4)))
+    inp = synth.tiny_inputs(wl, tag=200 + L)
+    q, K, _ = _upload(inp, dev)
+    ws = sg.make_workspace(Hq, Hkv, L, W, dev)
+    out = torch.empty((Hkv, L), dtype=torch.float32, device=dev)
+    sg.sgdkv_score(q, K, W, pool, out, ws)
+    torch.cuda.synchronize()
+    assert sg.sgdkv_last_error(ws) == sg.OK
+    raw = O.window_scores(inp["q"], inp["K"])
+    exp = O.max_pool(raw, pool)
+    got = out.cpu().numpy()
+    ok = _within(got, exp)
+    assert ok.all(), f"{(~ok).sum()} of {ok.size} off; worst {np.max(np.abs(got - exp))}"
+
+
+def _tie_heavy_scores(rng, Hkv, L):
+    return (rng.integers(0, 6, size=(Hkv, L)) * 0.125).astype(np.float32)
+
+
+COMPACT_CASES = [
+    # Hkv, L, n_sink, n_recent, budget rule
+    (4, 4096, 64, 64, "quarter"),
+    (2, 1000, 16, 16, "random"),
+    (3, 777, 0, 0, "random"),
+    (2, 300, 150, 150, "all"),        # no middle at all
+    (2, 5000, 10, 20, "floor"),       # nothing selected from the middle
+    (2, 5000, 10, 20, "full"),        # the whole middle selected
+    (5, 9000, 100, 28, "random"),     # several selection chunks, ragged tail
+    (1, 1, 0, 0, "full"),
+]
+
+
+def _budgets_for(rule, rng, Hkv, L, n_sink, n_recent):
+    lo, hi = n_sink + n_recent, L
+    if rule == "quarter":
+        return np.full(Hkv, max(lo, L // 4), np.int64)
+    if rule == "all" or rule == "full":
+        return np.full(Hkv, hi, np.int64)
+    if rule == "floor":
+        return np.full(Hkv, lo, np.int64)
+    return rng.integers(lo, hi + 1, size=Hkv).astype(np.int64)
+
+
+@pytest.mark.parametrize("Hkv,L,n_sink,n_recent,rule", COMPACT_CASES)
+@pytest.mark.parametrize("ties", [False, True])
+def test_compact_parity_identical_scores(dev, Hkv, L, n_sink, n_recent, rule, ties):
+    rng = np.random.default_rng(L * 7 + Hkv + int(ties))
+    scores = _tie_heavy_scores(rng, Hkv, L) if ties else rng.random((Hkv, L)).astype(np.float32)
+    K = synth.bf16_round(rng.standard_normal((Hkv, L, 128), dtype=np.float32))
+    V = synth.bf16_round(rng.standard_normal((Hkv, L, 128), dtype=np.float32))
+    b = _budgets_for(rule, rng, Hkv, L, n_sink, n_recent)
+    total = int(b.sum())
+    ws = sg.make_workspace(Hkv, Hkv, L, 32, dev) if L >= 32 else sg.make_workspace(1, 1, 32, 32, dev)
+    Kt, Vt = synth.to_torch_bf16(K, dev), synth.to_torch_bf16(V, dev)
+    st = torch.from_numpy(scores).to(dev)
+    idx = torch.full((max(total, 1),), -1, dtype=torch.int32, device=dev)
+    cu = torch.full((Hkv + 1,), -1, dtype=torch.int32, device=dev)
+    ko = torch.zeros((max(total, 1), 128), dtype=torch.bfloat16, device=dev)
+    vo = torch.zeros((max(total, 1), 128), dtype=torch.bfloat16, device=dev)
+    for _ in range(2):       # the same workspace twice in a row
+        sg.sgdkv_compact(Kt, Vt, st, b, n_sink, n_recent, idx, cu, ko, vo, ws)
+        torch.cuda.synchronize()
+        assert sg.sgdkv_last_error(ws) == sg.OK
+        e_idx, e_cu = O.select_indices(scores, b, n_sink, n_recent)
+        assert np.array_equal(cu.cpu().numpy(), e_cu)
+        assert np.array_equal(idx[:total].cpu().numpy(), e_idx)
+        e_ko, e_vo = O.gather(K, V, e_idx, e_cu)
+        assert np.array_equal(synth.from_torch_bf16(ko[:total]), e_ko)
+        assert np.array_equal(synth.from_torch_bf16(vo[:total]), e_vo)
+
+
+def _check_end_to_end(inp, out, budgets, n_sink, n_recent, pool):
+    raw = O.window_scores(inp["q"], inp["K"])
+    exp = O.max_pool(raw, pool) if pool > 1 else raw
+    got = out["scores"].cpu().numpy()
+    ok = _within(got, exp)
+    assert ok.all(), f"{(~ok).sum()} scores off; worst {np.max(np.abs(got - exp))}"
+    g_idx = out["indices"].cpu().numpy()
+    g_cu = out["cu_seqlens"].cpu().numpy()
+    s_idx, s_cu = O.select_indices(got, budgets, n_sink, n_recent)
+    assert np.array_equal(g_cu, s_cu)
+    assert np.array_equal(g_idx, s_idx)
+    o_idx, o_cu = O.select_indices(exp, budgets, n_sink, n_recent)
+    for h in range(len(budgets)):
+        a = set(g_idx[g_cu[h]:g_cu[h + 1]].tolist())
+        b = set(o_idx[o_cu[h]:o_cu[h + 1]].tolist())
+        diff = np.array(sorted(a ^ b), dtype=np.int64)
+        if diff.size:
+            kept = np.array(sorted(b - set(range(n_sink)) - set(range(len(exp[h]) - n_recent,
+                                                                      len(exp[h])))))
+            tau = exp[h, kept].min() if kept.size else 0.0
+            assert np.all(np.abs(exp[h, diff] - tau) <= ATOL + RTOL * abs(tau))
+    ko, vo = O.gather(inp["K"], inp["V"], g_idx, g_cu)
+    assert np.array_equal(synth.from_torch_bf16(out["K_out"]), ko)
+    assert np.array_equal(synth.from_torch_bf16(out["V_out"]), vo)
+
+
+def test_compress_layer_small(dev):
+    wl = synth.tiny_workload(Hq=28, Hkv=4, d=128, L=5000, W=64, n_salient=32, floor=256)
+    inp = synth.tiny_inputs(wl, tag=300)
+    q, K, V = _upload(inp, dev)
+    b = np.array([1250, 700, 2400, 256], np.int64)
+    ws = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
+    out = sg.compress_layer_alloc(q, K, V, b, wl.W, 7, 128, 128, ws)
+    torch.cuda.synchronize()
+    assert sg.sgdkv_last_error(ws) == sg.OK
+    _check_end_to_end(inp, out, b, 128, 128, 7)
+
+
+@pytest.mark.parametrize("name", [w.name for w in configs.WORKLOADS])
+def test_full_size_layer(dev, name):
+    """One layer of each workload at full size, in the launch configuration the benchmark
+    times (sgdkv_compress_layer with the model-wide greedy allocation)."""
+    wl = configs.BY_NAME[name]
+    layer = wl.n_layers - 1
+    inp = synth.layer_inputs_host(wl, layer)
+    frac = 0.25 if 0.25 in wl.budget_fracs else wl.budget_fracs[0]
+    all_b = sg.sgdkv_allocate_budgets(synth.head_scores(wl), wl.L, wl.total_budget(frac), wl.floor)
+    b = all_b[layer * wl.Hkv:(layer + 1) * wl.Hkv]
+    n_sink, n_recent = configs.sink_recent_split(wl.floor)
+    q, K, V = _upload(inp, dev)
+    ws = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
+    out = sg.compress_layer_alloc(q, K, V, b, wl.W, wl.pool, n_sink, n_recent, ws)
+    torch.cuda.synchronize()
+    assert sg.sgdkv_last_error(ws) == sg.OK
+    _check_end_to_end(inp, out, b, n_sink, n_recent, wl.pool)
+    # planted keys (4 sinks + salient) survive whenever the middle budget has room
+    g_idx, g_cu = out["indices"].cpu().numpy(), out["cu_seqlens"].cpu().numpy()
+    for h in range(wl.Hkv):
+        if b[h] - wl.floor >= 7 * len(inp["planted"][h]):
+            kept = set(g_idx[g_cu[h]:g_cu[h + 1]].tolist())
+            assert set(inp["planted"][h].tolist()) <= kept
+
+
+def test_rejects_misaligned_pointer(dev):
+    wl = synth.tiny_workload(Hq=14, Hkv=2, L=512, W=32)
+    inp = synth.tiny_inputs(wl)
+    q, K, _ = _upload(inp, dev)
+    ws = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
+    big = torch.empty(2 * 512 + 1, dtype=torch.float32, device=dev)
+    with pytest.raises(sg.SgdkvError) as e:
+        sg.sgdkv_score(q, K, wl.W, 7, big[1:], ws)
+    assert e.value.status == sg.ERR_INVALID_ARG
