@@ -157,6 +157,15 @@ SGDKV_API sgdkv_status sgdkv_compress_layer(const void* q_win, const void* K, co
 SGDKV_API uint64_t sgdkv_launch_count(void);
 
 /*
+ * Test hook (no counterpart in the paper): sets the time bound, in nanoseconds, of every
+ * device-side wait in the scoring kernels (0 restores the default of 2 s), and flags:
+ * bit 0 makes the scoring kernels' MMA issuer first wait on a barrier nothing signals, so
+ * that the wait runs out, SGDKV_ERR_TIMEOUT is recorded and the kernels drain and exit.
+ * Process-wide; affects launches issued after the call.  Not thread-safe.
+ */
+SGDKV_API void sgdkv_debug_set_score_hooks(uint32_t flags, uint64_t wait_ns);
+
+/*
  * Synchronises `stream`, then returns and clears the first device-side failure recorded
  * in `workspace` since the last call (SGDKV_OK if none), or SGDKV_ERR_CUDA if the stream
  * itself reports an error.

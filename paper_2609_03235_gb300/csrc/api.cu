@@ -36,7 +36,7 @@ WsLayout workspace_layout(int32_t Hkv, int64_t L) {
   w.chunk_cnt = take(H * n_sel_chunks * sizeof(uint2));
   w.lse = take(H * kMaxRows * sizeof(float));
   w.partial = take(H * size_t(kMaxScoreParts) * kMaxRows * sizeof(float2));
-  w.raw = take(H * size_t(L) * sizeof(float));
+  w.raw = take(2 * H * size_t(L) * sizeof(float));
   w.pooled = take(H * size_t(L) * sizeof(float));
   w.total = off;
   return w;
@@ -131,6 +131,11 @@ const char* sgdkv_status_string(int status) {
 int sgdkv_version(void) { return 100; }
 
 uint64_t sgdkv_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+void sgdkv_debug_set_score_hooks(uint32_t flags, uint64_t wait_ns) {
+  g_score_flags = flags;
+  g_score_wait_ns = wait_ns > 0 ? wait_ns : 2000000000ull;
+}
 
 size_t sgdkv_workspace_bytes(int32_t Hq, int32_t Hkv, int64_t L, int32_t d, int32_t W) {
   if (check_score_shape(Hq, Hkv, L, d, W) != SGDKV_OK) return 0;

@@ -1,0 +1,659 @@
+// Window scoring on the 5th-generation tensor cores (tcgen05 + TMEM + TMA), sm_103a.
+//
+// Computes the cumulative window attention of Section 3.3 / Section 5 (SnapKV-style):
+//   raw[h][j] = sum_{g<G} sum_{w<W} softmax_j(q[h*G+g][w] . K[h][j] / sqrt(d)),
+// window row w seeing keys j <= L - W + w.  With t_rj = (q_r . k_j) * log2(e)/sqrt(d) and
+// the G*W window rows r = g*W + w of KV head h (contiguous in q_win):
+//
+//   pass 1 (score_pass1_tc): D[r][j] = Q_h K_tile^T on the tensor cores (rows on TMEM
+//     lanes, keys on columns); every epilogue thread owns one window row and keeps an
+//     online (max m_r, sum Z_r = sum 2^(t_rj - m_r)) over the keys of its CTA's range;
+//     the per-CTA partials go to the workspace.
+//   pass 2 (score_pass2_tc): merges the partials into lse_r = m_r + log2 Z_r, then
+//     D[j][r] = K_tile Q_h^T (keys on TMEM lanes, rows on columns); every epilogue thread
+//     owns one key and sums 2^(t_rj - lse_r) over the window rows (two warps per key, each
+//     half of the rows, written to two halves of the raw buffer).
+//   pool (maxpool_sum_kernel): scores = max-pool of (raw half 0 + raw half 1).
+//
+// CTA roles (320 threads): warp 0 lane 0 issues TMA loads (Q once, K tiles of 128 keys
+// through a ring of shared-memory stages); warp 1 allocates the 512 TMEM columns and its
+// lane 0 issues the MMAs; warps 2..9 are the epilogue (two per TMEM lane quarter).  Each
+// CTA owns one KV head and a contiguous range of key tiles.  Every wait on an mbarrier is
+// bounded in time: on expiry the kernel records SGDKV_ERR_TIMEOUT, all roles leave their
+// loops, in-flight copies and MMAs are drained (again bounded) and TMEM is freed.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "sgdkv_internal.cuh"
+
+namespace sgdkv {
+namespace {
+
+constexpr int kThreads = 320;
+constexpr int kEpiWarps = 8;
+constexpr int kTileKeys = 128;
+constexpr uint32_t kTmemCols = 512;
+constexpr int kStageBytes = kTileKeys * 256;      // 32 KB: two 128-byte column halves
+constexpr int kHalfBytes = kTileKeys * 128;       // 16 KB
+constexpr int kNumBars = 15;   // kfull[4] kempty[4] tfull[2] tempty[2] qfull drain never
+constexpr int kCtlBytes = 128;                    // barriers + TMEM address + abort flag
+constexpr uint32_t kFlagStallMma = 1u;            // test hook: MMA thread waits on `never`
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr uint64_t kDrainNs = 1000000000ull;      // bound on cleanup waits after an abort
+
+struct TcParams {
+  int Hkv, G, W, GW;
+  int64_t L;
+  int T;          // key tiles (of 128) per head
+  int cph;        // CTAs per head
+  int nrt;        // window-row tiles of 128 (pass 1) = ceil(GW / 128)
+  int nstages;    // K ring depth
+  int nparts;     // pass 2: partial slots per head written by pass 1
+  int ppc;        // pass 1: partial slots per CTA
+  float scale2;   // log2(e) / sqrt(d)
+  uint64_t wait_ns;
+  uint32_t flags;
+};
+
+// ---------------------------------------------------------------------------------------
+// PTX wrappers
+// ---------------------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Waits for the phase of `bar` with the given parity; false if the CTA aborted or the wait
+// ran past limit_ns (then the timeout is recorded and the CTA-wide abort flag raised).
+__device__ __noinline__ bool bwait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                   uint64_t limit_ns, uint32_t* status) {
+  if (mbar_try(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try(bar, parity)) return true;
+    if ((it & 15u) == 0) {
+      if (*abort_flag) return false;
+      if (global_ns() - t0 > limit_ns) {
+        record_error(status, SGDKV_ERR_TIMEOUT);
+        *abort_flag = 1;
+        return false;
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of 128 bytes in
+// 8-row atoms of 1024 bytes (the layout a TMA box {64 bf16, rows} with SWIZZLE_128B writes).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= uint64_t((saddr >> 4) & 0x3FFFu);
+  d |= uint64_t(1) << 16;              // leading-dimension offset (unused for this layout)
+  d |= uint64_t(1024 >> 4) << 32;      // stride between 8-row groups
+  d |= uint64_t(1) << 46;              // descriptor version
+  d |= uint64_t(2) << 61;              // SWIZZLE_128B
+  return d;
+}
+// Instruction descriptor, kind::f16: bf16 A and B (K-major), fp32 accumulator, M x N.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(N >> 3) << 17) | (uint32_t(M >> 4) << 24);
+}
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+#define SGDKV_LD_REGS32(r)                                                                   \
+  "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),       \
+      "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), \
+      "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),          \
+      "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),          \
+      "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+
+// 32 consecutive fp32 TMEM columns of this thread's lane (32x32b shape, x32).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : SGDKV_LD_REGS32(r)
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// ---------------------------------------------------------------------------------------
+// Shared pieces of both passes
+// ---------------------------------------------------------------------------------------
+struct Smem {
+  uint8_t* q;          // 2 halves x qrows x 128 B
+  uint8_t* k;          // nstages x 32 KB
+  uint64_t* bars;      // kNumBars
+  uint32_t* tmem_slot;
+  int* abort_flag;
+  float* tail;         // pass 2: lse2[kMaxRows]
+  int qrows;
+};
+
+__device__ __forceinline__ Smem carve(uint8_t* base, int qrows, int nstages) {
+  Smem s;
+  s.qrows = qrows;
+  s.q = base;
+  s.k = base + 2 * qrows * 128;
+  uint8_t* ctl = s.k + nstages * kStageBytes;
+  s.bars = reinterpret_cast<uint64_t*>(ctl);
+  s.tmem_slot = reinterpret_cast<uint32_t*>(ctl + kNumBars * 8);
+  s.abort_flag = reinterpret_cast<int*>(ctl + kNumBars * 8 + 4);
+  s.tail = reinterpret_cast<float*>(ctl + kCtlBytes);
+  return s;
+}
+__device__ __forceinline__ uint32_t bar_kfull(const Smem& s, int i) { return smem_u32(s.bars + i); }
+__device__ __forceinline__ uint32_t bar_kempty(const Smem& s, int i) { return smem_u32(s.bars + 4 + i); }
+__device__ __forceinline__ uint32_t bar_tfull(const Smem& s, int i) { return smem_u32(s.bars + 8 + i); }
+__device__ __forceinline__ uint32_t bar_tempty(const Smem& s, int i) { return smem_u32(s.bars + 10 + i); }
+__device__ __forceinline__ uint32_t bar_qfull(const Smem& s) { return smem_u32(s.bars + 12); }
+__device__ __forceinline__ uint32_t bar_drain(const Smem& s) { return smem_u32(s.bars + 13); }
+__device__ __forceinline__ uint32_t bar_never(const Smem& s) { return smem_u32(s.bars + 14); }
+
+// Barrier init, TMEM allocation; returns the TMEM base address (all threads).
+__device__ __forceinline__ uint32_t setup(const Smem& s, int nstages) {
+  const int warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < nstages; ++i) {
+      mbar_init(bar_kfull(s, i), 1);
+      mbar_init(bar_kempty(s, i), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(bar_tfull(s, i), 1);
+      mbar_init(bar_tempty(s, i), kEpiWarps);
+    }
+    mbar_init(bar_qfull(s), 1);
+    mbar_init(bar_drain(s), 1);
+    mbar_init(bar_never(s), 1);
+    *s.abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(s.tmem_slot)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  return *s.tmem_slot;
+}
+
+__device__ __forceinline__ void teardown(uint32_t tmem) {
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if ((threadIdx.x >> 5) == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(kTmemCols)
+                 : "memory");
+  }
+}
+
+// TMA producer (one thread): Q rows of head h once, then the CTA's key tiles.
+__device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMap* tm_k,
+                        const TcParams& p, int h, int t0, int ntiles, uint32_t* status) {
+  volatile int* ab = s.abort_flag;
+  const int qboxes = s.qrows / 128;
+  mbar_expect_tx(bar_qfull(s), uint32_t(2 * s.qrows * 128));
+  for (int c = 0; c < 2; ++c)
+    for (int b = 0; b < qboxes; ++b)
+      tma_load_2d(smem_u32(s.q + c * s.qrows * 128 + b * kHalfBytes), tm_q, 64 * c,
+                  h * p.GW + 128 * b, bar_qfull(s));
+  int issued[4] = {0, 0, 0, 0};
+  for (int n = 0; n < ntiles; ++n) {
+    const int st = n % p.nstages;
+    const int use = n / p.nstages;
+    if (!bwait(bar_kempty(s, st), (use & 1) ^ 1, ab, p.wait_ns, status)) break;
+    mbar_expect_tx(bar_kfull(s, st), kStageBytes);
+    const int row = int(int64_t(h) * p.L + int64_t(t0 + n) * kTileKeys);
+    for (int c = 0; c < 2; ++c)
+      tma_load_2d(smem_u32(s.k + st * kStageBytes + c * kHalfBytes), tm_k, 64 * c, row,
+                  bar_kfull(s, st));
+    issued[st] = use + 1;
+  }
+  if (*ab) {
+    // Drain: every copy this thread started must have landed before the CTA exits.
+    volatile int no_abort = 0;
+    bwait(bar_qfull(s), 0, &no_abort, kDrainNs, status);
+    for (int st = 0; st < p.nstages; ++st)
+      if (issued[st] > 0) bwait(bar_kfull(s, st), (issued[st] - 1) & 1, &no_abort, kDrainNs, status);
+  }
+}
+
+// MMA thread, start of its work: the optional stall hook (a wait on a barrier nothing
+// arrives on, to exercise the timeout path), then the wait for the Q rows.
+__device__ bool mma_start(const Smem& s, const TcParams& p, uint32_t* status) {
+  volatile int* ab = s.abort_flag;
+  if ((p.flags & kFlagStallMma) && !bwait(bar_never(s), 0, ab, p.wait_ns, status)) return false;
+  return bwait(bar_qfull(s), 0, ab, p.wait_ns, status);
+}
+
+// MMA thread, after an abort: a commit arrives on `drain` once every MMA this thread issued
+// has completed, so TMEM is not released under a running MMA.
+__device__ void mma_drain(const Smem& s, uint32_t* status) {
+  umma_commit(bar_drain(s));
+  volatile int no_abort = 0;
+  bwait(bar_drain(s), 0, &no_abort, kDrainNs, status);
+}
+
+// ---------------------------------------------------------------------------------------
+// Pass 1: per window row, online (max, sum of 2^(t - max)) over the CTA's key range
+// ---------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads, 1)
+score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+               TcParams p, Ws ws) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  if (smem_u32(smem_raw) & 1023u) {
+    if (threadIdx.x == 0) record_error(ws.status, SGDKV_ERR_INTERNAL);
+    return;
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.x / p.cph, ci = blockIdx.x % p.cph;
+  const int t0 = int(int64_t(ci) * p.T / p.cph);
+  const int t1 = int(int64_t(ci + 1) * p.T / p.cph);
+  const int ntiles = t1 - t0;
+  const Smem s = carve(smem_raw, p.nrt * 128, p.nstages);
+  const uint32_t tmem = setup(s, p.nstages);
+  volatile int* ab = s.abort_flag;
+  const int sub = p.nrt >= 3 ? 2 : 1;          // MMA sub-chunks per 128-key tile
+  const int nsub = kTileKeys / sub;            // keys per sub-chunk (MMA N)
+
+  if (warp == 0) {
+    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, t0, ntiles, ws.status);
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16(128, nsub);
+      bool ok = mma_start(s, p, ws.status);
+      const uint32_t q0 = smem_u32(s.q), qhalf = uint32_t(s.qrows * 128);
+      for (int n = 0; ok && n < ntiles; ++n) {
+        const int st = n % p.nstages;
+        if (!(ok = bwait(bar_kfull(s, st), (n / p.nstages) & 1, ab, p.wait_ns, ws.status))) break;
+        tc_fence_after();
+        const uint32_t k0 = smem_u32(s.k + st * kStageBytes);
+        for (int j = 0; j < sub; ++j) {
+          const int u = n * sub + j, slot = u & 1;
+          if (!(ok = bwait(bar_tempty(s, slot), ((u >> 1) & 1) ^ 1, ab, p.wait_ns, ws.status)))
+            break;
+          tc_fence_after();
+          for (int rt = 0; rt < p.nrt; ++rt)
+            for (int k = 0; k < 8; ++k) {
+              const uint32_t koff = uint32_t((k & 3) * 32), half = uint32_t(k >> 2);
+              const uint64_t a = sw128_desc(q0 + half * qhalf + uint32_t(rt) * kHalfBytes + koff);
+              const uint64_t b = sw128_desc(k0 + half * kHalfBytes + uint32_t(j * nsub) * 128 + koff);
+              umma_bf16(tmem + uint32_t(slot * 256 + rt * nsub), a, b, idesc, k > 0 ? 1u : 0u);
+            }
+          umma_commit(bar_tfull(s, slot));
+        }
+        if (ok) umma_commit(bar_kempty(s, st));
+      }
+      if (!ok) mma_drain(s, ws.status);
+    }
+  } else {
+    const int ew = warp - 2, q = warp & 3, g = ew >> 2;
+    const bool row_split = p.nrt >= 2;
+    float m[2] = {-INFINITY, -INFINITY}, Z[2] = {0.f, 0.f};
+    const int64_t lim_base = p.L - p.W;
+    bool ok = true;
+    for (int n = 0; ok && n < ntiles; ++n) {
+      const int64_t key0 = int64_t(t0 + n) * kTileKeys;
+      for (int j = 0; j < sub; ++j) {
+        const int u = n * sub + j, slot = u & 1;
+        if (!(ok = bwait(bar_tfull(s, slot), (u >> 1) & 1, ab, p.wait_ns, ws.status))) break;
+        tc_fence_after();
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+          const int rt = row_split ? g + 2 * i : 0;
+          const int r0 = rt * 128 + 32 * q;
+          // warp-uniform: row tile present and not padding
+          if (rt >= p.nrt || (!row_split && i > 0) || r0 >= p.GW) continue;
+          const int64_t lim = lim_base + (r0 + lane) % p.W;
+          const int c_lo = row_split ? 0 : g * (nsub / 2);
+          const int c_hi = row_split ? nsub : c_lo + nsub / 2;
+          for (int c0 = c_lo; c0 < c_hi; c0 += 32) {
+            uint32_t v[32];
+            tmem_ld32(tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256 + rt * nsub + c0), v);
+            tmem_wait_ld();
+            const int64_t kb = key0 + j * nsub + c0;
+            float x[32];
+            float mx = -INFINITY;
+            if (kb + 31 > lim_base) {
+#pragma unroll
+              for (int e = 0; e < 32; ++e) {
+                x[e] = (kb + e <= lim) ? __uint_as_float(v[e]) : -INFINITY;
+                mx = fmaxf(mx, x[e]);
+              }
+            } else {
+#pragma unroll
+              for (int e = 0; e < 32; ++e) {
+                x[e] = __uint_as_float(v[e]);
+                mx = fmaxf(mx, x[e]);
+              }
+            }
+            if (mx == -INFINITY) continue;
+            const float mn = fmaxf(m[i], mx * p.scale2);
+            if (mn > m[i]) {
+              Z[i] = (m[i] == -INFINITY) ? 0.f : Z[i] * ex2(m[i] - mn);
+              m[i] = mn;
+            }
+            float zc = 0.f;
+#pragma unroll
+            for (int e = 0; e < 32; ++e) zc += ex2(fmaf(x[e], p.scale2, -m[i]));
+            Z[i] += zc;
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar_tempty(s, slot));
+      }
+    }
+    if (ok) {
+      const int slot_base = ci * p.ppc + (row_split ? 0 : g);
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        const int rt = row_split ? g + 2 * i : 0;
+        const int r = rt * 128 + 32 * q + lane;
+        if (rt >= p.nrt || (!row_split && i > 0) || rt * 128 + 32 * q >= p.GW) continue;
+        ws.partial[(int64_t(h) * kMaxScoreParts + slot_base) * kMaxRows + r] = make_float2(m[i], Z[i]);
+      }
+    }
+  }
+  teardown(tmem);
+}
+
+// ---------------------------------------------------------------------------------------
+// Pass 2: per key, sum over window rows of 2^(t - lse)
+// ---------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads, 1)
+score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+               TcParams p, Ws ws) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  if (smem_u32(smem_raw) & 1023u) {
+    if (threadIdx.x == 0) record_error(ws.status, SGDKV_ERR_INTERNAL);
+    return;
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.x / p.cph, ci = blockIdx.x % p.cph;
+  const int t0 = int(int64_t(ci) * p.T / p.cph);
+  const int t1 = int(int64_t(ci + 1) * p.T / p.cph);
+  const int ntiles = t1 - t0;
+  const Smem s = carve(smem_raw, p.nrt * 128, p.nstages);
+  float* lse2 = s.tail;                          // [kMaxRows]
+  const uint32_t tmem = setup(s, p.nstages);
+  volatile int* ab = s.abort_flag;
+  const int nch = p.GW > 256 ? 2 : 1;            // N chunks of the window rows per tile
+  const int nn = p.GW / nch;                     // MMA N
+
+  if (warp == 0) {
+    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, t0, ntiles, ws.status);
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16(128, nn);
+      bool ok = mma_start(s, p, ws.status);
+      const uint32_t q0 = smem_u32(s.q), qhalf = uint32_t(s.qrows * 128);
+      for (int n = 0; ok && n < ntiles; ++n) {
+        const int st = n % p.nstages;
+        if (!(ok = bwait(bar_kfull(s, st), (n / p.nstages) & 1, ab, p.wait_ns, ws.status))) break;
+        tc_fence_after();
+        const uint32_t k0 = smem_u32(s.k + st * kStageBytes);
+        for (int c = 0; c < nch; ++c) {
+          const int u = n * nch + c, slot = u & 1;
+          if (!(ok = bwait(bar_tempty(s, slot), ((u >> 1) & 1) ^ 1, ab, p.wait_ns, ws.status)))
+            break;
+          tc_fence_after();
+          for (int k = 0; k < 8; ++k) {
+            const uint32_t koff = uint32_t((k & 3) * 32), half = uint32_t(k >> 2);
+            const uint64_t a = sw128_desc(k0 + half * kHalfBytes + koff);
+            const uint64_t b = sw128_desc(q0 + half * qhalf + uint32_t(c * nn) * 128 + koff);
+            umma_bf16(tmem + uint32_t(slot * 256), a, b, idesc, k > 0 ? 1u : 0u);
+          }
+          umma_commit(bar_tfull(s, slot));
+        }
+        if (ok) umma_commit(bar_kempty(s, st));
+      }
+      if (!ok) mma_drain(s, ws.status);
+    }
+  } else {
+    const int ew = warp - 2, q = warp & 3, g = ew >> 2;
+    // Merge pass-1 partials of every window row into lse2 (log2 units).
+    for (int r = ew * 32 + lane; r < p.GW; r += kEpiWarps * 32) {
+      const float2* pp = ws.partial + int64_t(h) * kMaxScoreParts * kMaxRows + r;
+      float M = -INFINITY;
+      for (int i = 0; i < p.nparts; ++i) M = fmaxf(M, pp[int64_t(i) * kMaxRows].x);
+      float S = 0.f;
+      for (int i = 0; i < p.nparts; ++i) {
+        const float2 v = pp[int64_t(i) * kMaxRows];
+        if (v.x != -INFINITY) S += v.y * ex2(v.x - M);
+      }
+      lse2[r] = M + log2f(S);
+    }
+    asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+    // columns of each N chunk handled by this warp group: split at a multiple of 16
+    const int split = ((nn / 2 + 15) / 16) * 16;
+    const int c_lo = g ? split : 0;
+    const int half_cols = g ? nn - split : split;
+    float* raw_out = ws.raw + int64_t(g) * p.Hkv * p.L + int64_t(h) * p.L;
+    const int64_t lim_base = p.L - p.W;
+    bool ok = true;
+    for (int n = 0; ok && n < ntiles; ++n) {
+      const int64_t key0 = int64_t(t0 + n) * kTileKeys;
+      const int64_t j = key0 + 32 * q + lane;
+      const bool masked = key0 + kTileKeys - 1 > lim_base;
+      float acc = 0.f;
+      for (int c = 0; c < nch; ++c) {
+        const int u = n * nch + c, slot = u & 1;
+        if (!(ok = bwait(bar_tfull(s, slot), (u >> 1) & 1, ab, p.wait_ns, ws.status))) break;
+        tc_fence_after();
+        const uint32_t tbase = tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256);
+        for (int c0 = 0; c0 < half_cols; c0 += 32) {
+          uint32_t v[32];
+          const bool full = c0 + 32 <= half_cols;
+          if (full) tmem_ld32(tbase + uint32_t(c_lo + c0), v);
+          else tmem_ld16(tbase + uint32_t(c_lo + c0), v);
+          tmem_wait_ld();
+          const int nv = full ? 32 : 16;
+          const int rbase = c * nn + c_lo + c0;
+          if (!masked) {
+            if (full) {
+#pragma unroll
+              for (int e = 0; e < 32; ++e)
+                acc += ex2(fmaf(__uint_as_float(v[e]), p.scale2, -lse2[rbase + e]));
+            } else {
+#pragma unroll
+              for (int e = 0; e < 16; ++e)
+                acc += ex2(fmaf(__uint_as_float(v[e]), p.scale2, -lse2[rbase + e]));
+            }
+          } else {
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+              const int r = rbase + e;
+              if (e < nv && j <= lim_base + r % p.W)
+                acc += ex2(fmaf(__uint_as_float(v[e]), p.scale2, -lse2[r]));
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar_tempty(s, slot));
+      }
+      if (ok && j < p.L) raw_out[j] = acc;
+    }
+  }
+  teardown(tmem);
+}
+
+// scores = max-pool over [j - radius, j + radius] (clipped) of raw0 + raw1.
+__global__ void maxpool_sum_kernel(const float* __restrict__ raw, float* __restrict__ out,
+                                   int64_t L, int64_t n, int radius) {
+  const int64_t t = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (t >= n) return;
+  const int64_t j = t % L;
+  const float* r0 = raw + (t - j);
+  const float* r1 = r0 + n;
+  float m = r0[j] + r1[j];
+  for (int s = 1; s <= radius; ++s) {
+    if (j - s >= 0) m = fmaxf(m, r0[j - s] + r1[j - s]);
+    if (j + s < L) m = fmaxf(m, r0[j + s] + r1[j + s]);
+  }
+  out[t] = m;
+}
+
+// ---------------------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------------------
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  }
+  return fn;
+}
+
+// 2-D bf16 map over a [rows][128] row-major matrix, box {64 columns, 128 rows}, 128B swizzle.
+bool make_map(CUtensorMap* map, const void* base, uint64_t rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[2] = {cuuint64_t(kD), cuuint64_t(rows)};
+  const cuuint64_t strides[1] = {cuuint64_t(kD * 2)};
+  const cuuint32_t box[2] = {64, 128};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int sm_count() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 148;
+  return n;
+}
+
+}  // namespace
+
+uint64_t g_score_wait_ns = 2000000000ull;
+uint32_t g_score_flags = 0;
+
+cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
+                         int64_t L, int W, int pool, float* scores_out, const Ws& ws,
+                         cudaStream_t stream) {
+  TcParams p{};
+  p.Hkv = Hkv;
+  p.G = Hq / Hkv;
+  p.W = W;
+  p.GW = p.G * W;
+  p.L = L;
+  p.T = int(ceil_div(L, kTileKeys));
+  const int nsm = sm_count();
+  p.cph = nsm / Hkv;
+  if (p.cph < 1) p.cph = 1;
+  if (p.cph > p.T) p.cph = p.T;
+  p.nrt = int(ceil_div(p.GW, 128));
+  p.nstages = p.GW > 256 ? 2 : 4;
+  p.ppc = p.nrt >= 2 ? 1 : 2;
+  p.nparts = p.cph * p.ppc;
+  if (p.nparts > kMaxScoreParts) return cudaErrorInvalidConfiguration;
+  p.scale2 = kLog2e / sqrtf(float(kD));
+  p.wait_ns = g_score_wait_ns;
+  p.flags = g_score_flags;
+
+  CUtensorMap tm_q, tm_k;
+  if (!make_map(&tm_q, q, uint64_t(Hq) * W) || !make_map(&tm_k, K, uint64_t(Hkv) * L))
+    return cudaErrorInvalidValue;
+  const size_t base = size_t(2) * p.nrt * 128 * 128 + size_t(p.nstages) * kStageBytes + kCtlBytes;
+  const size_t smem1 = base;
+  const size_t smem2 = base + kMaxRows * sizeof(float);
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(score_pass1_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                int(smem1))) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(score_pass2_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                int(smem2))) != cudaSuccess)
+    return e;
+  const int grid = Hkv * p.cph;
+  score_pass1_tc<<<grid, kThreads, smem1, stream>>>(tm_q, tm_k, p, ws);
+  score_pass2_tc<<<grid, kThreads, smem2, stream>>>(tm_q, tm_k, p, ws);
+  const int64_t n = int64_t(Hkv) * L;
+  maxpool_sum_kernel<<<unsigned(ceil_div(n, 256)), 256, 0, stream>>>(ws.raw, scores_out, L, n,
+                                                                    pool / 2);
+  note_launches(3);
+  return cudaGetLastError();
+}
+
+}  // namespace sgdkv

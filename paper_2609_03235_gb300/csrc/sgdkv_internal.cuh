@@ -13,7 +13,7 @@ namespace sgdkv {
 
 constexpr int kD = SGDKV_HEAD_DIM;     // head dim supported by v1
 constexpr int kMaxRows = 512;          // G*W limit (window rows of one KV head)
-constexpr int kMaxScoreParts = 256;    // pass-1 partial (m, Z) slots per KV head
+constexpr int kMaxScoreParts = 320;    // pass-1 partial (m, Z) slots per KV head
 constexpr int kSelChunk = 4096;        // selection elements per CTA
 constexpr int kSelThreads = 256;       // threads per selection CTA (16 elements each)
 constexpr int kSelPerThread = kSelChunk / kSelThreads;
@@ -48,7 +48,7 @@ struct Ws {
   uint2* chunk_cnt;      // [Hkv][n_sel_chunks] (kept non-ties, ties) per selection chunk
   float* lse;            // [Hkv][kMaxRows] per window row: log2 of its softmax normaliser
   float2* partial;       // [Hkv][kMaxScoreParts][kMaxRows] per-part (max, sum) in log2 units
-  float* raw;            // [Hkv][L] window scores before pooling
+  float* raw;            // [2][Hkv][L] window scores before pooling, as two partial sums
   float* pooled;         // [Hkv][L] pooled scores (compress_layer scratch)
 };
 
@@ -67,6 +67,10 @@ __device__ __forceinline__ void record_error(uint32_t* status, uint32_t code) {
 
 // Counts kernel launches issued by the library (sgdkv_launch_count).
 void note_launches(int n);
+
+// Scorer wait bound and test-hook flags (sgdkv_debug_set_score_hooks).
+extern uint64_t g_score_wait_ns;
+extern uint32_t g_score_flags;
 
 // Launchers (each returns cudaGetLastError() after its launches).
 cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,

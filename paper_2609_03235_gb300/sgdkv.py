@@ -19,7 +19,7 @@ OK, ERR_INVALID_ARG, ERR_INFEASIBLE_BUDGET, ERR_WORKSPACE, ERR_CUDA, ERR_TIMEOUT
 ALLOC_GREEDY, ALLOC_PROPORTIONAL, ALLOC_THRESHOLD = 0, 1, 2
 EXPORTED = ("sgdkv_status_string", "sgdkv_version", "sgdkv_allocate_budgets",
             "sgdkv_workspace_bytes", "sgdkv_score", "sgdkv_compact", "sgdkv_compress_layer",
-            "sgdkv_last_error", "sgdkv_launch_count")
+            "sgdkv_last_error", "sgdkv_launch_count", "sgdkv_debug_set_score_hooks")
 
 
 class LibraryMissing(RuntimeError):
@@ -62,6 +62,8 @@ def lib():
         L.sgdkv_last_error.restype = ctypes.c_int
         L.sgdkv_last_error.argtypes = [_P, _P]
         L.sgdkv_launch_count.restype = ctypes.c_uint64
+        L.sgdkv_debug_set_score_hooks.restype = None
+        L.sgdkv_debug_set_score_hooks.argtypes = [ctypes.c_uint32, ctypes.c_uint64]
         _lib = L
     return _lib
 
@@ -153,6 +155,10 @@ def sgdkv_compress_layer(q_win, K, V, budgets, W: int, pool: int, n_sink: int, n
 
 def sgdkv_launch_count() -> int:
     return int(lib().sgdkv_launch_count())
+
+
+def sgdkv_debug_set_score_hooks(flags: int, wait_ns: int = 0) -> None:
+    lib().sgdkv_debug_set_score_hooks(int(flags), int(wait_ns))
 
 
 def sgdkv_last_error(workspace, stream=None) -> int:

@@ -42,6 +42,8 @@ SCORE_SHAPES = [
     (7, 1, 32, 32),        # L == W: every key is a window key
     (8, 8, 640, 32),
     (28, 4, 129, 64),
+    (9, 1, 1000, 32),      # G*W = 288: three row tiles, N chunks of 144 split 80 / 64
+    (28, 4, 20000, 64),    # several key tiles per CTA
 ]
 
 
