@@ -157,6 +157,12 @@ SGDKV_API sgdkv_status sgdkv_compress_layer(const void* q_win, const void* K, co
 SGDKV_API uint64_t sgdkv_launch_count(void);
 
 /*
+ * Diagnostics: text of the last CUDA runtime error this library saw on the calling thread
+ * ("no error" if none).  Explains an SGDKV_ERR_CUDA result.  Never NULL.
+ */
+SGDKV_API const char* sgdkv_last_cuda_error_string(void);
+
+/*
  * Test hook (no counterpart in the paper): sets the time bound, in nanoseconds, of every
  * device-side wait in the scoring kernels (0 restores the default of 2 s), and flags:
  * bit 0 makes the scoring kernels' MMA issuer first wait on a barrier nothing signals, so

@@ -26,17 +26,18 @@ WsLayout workspace_layout(int32_t Hkv, int64_t L) {
     off = align256(off + bytes);
     return at;
   };
+  const size_t HM = SGDKV_MAX_KV_HEADS;
   const size_t H = size_t(Hkv);
   const size_t n_sel_chunks = size_t(ceil_div(L, kSelChunk));
+  // fixed control block
   w.status = take(256);
-  w.merge_cnt = take(H * sizeof(uint32_t));
-  w.sel = take(H * sizeof(SelState));
-  w.hist = take(H * 256 * sizeof(uint32_t));
-  w.sel_cnt = take(H * sizeof(uint32_t));
+  w.hist = take(HM * kRadixBins * sizeof(uint32_t));
+  w.sel_cnt = take(HM * sizeof(uint32_t));
+  w.sel = take(HM * sizeof(SelState));
+  // shape-dependent scratch
   w.chunk_cnt = take(H * n_sel_chunks * sizeof(uint2));
-  w.lse = take(H * kMaxRows * sizeof(float));
   w.partial = take(H * size_t(kMaxScoreParts) * kMaxRows * sizeof(float2));
-  w.raw = take(2 * H * size_t(L) * sizeof(float));
+  w.raw = take(4 * H * size_t(L) * sizeof(float));
   w.pooled = take(H * size_t(L) * sizeof(float));
   w.total = off;
   return w;
@@ -46,12 +47,10 @@ Ws workspace_view(void* base, const WsLayout& lay) {
   char* b = static_cast<char*>(base);
   Ws ws;
   ws.status = reinterpret_cast<uint32_t*>(b + lay.status);
-  ws.merge_cnt = reinterpret_cast<uint32_t*>(b + lay.merge_cnt);
-  ws.sel = reinterpret_cast<SelState*>(b + lay.sel);
   ws.hist = reinterpret_cast<uint32_t*>(b + lay.hist);
   ws.sel_cnt = reinterpret_cast<uint32_t*>(b + lay.sel_cnt);
+  ws.sel = reinterpret_cast<SelState*>(b + lay.sel);
   ws.chunk_cnt = reinterpret_cast<uint2*>(b + lay.chunk_cnt);
-  ws.lse = reinterpret_cast<float*>(b + lay.lse);
   ws.partial = reinterpret_cast<float2*>(b + lay.partial);
   ws.raw = reinterpret_cast<float*>(b + lay.raw);
   ws.pooled = reinterpret_cast<float*>(b + lay.pooled);
@@ -105,7 +104,13 @@ sgdkv_status build_head_table(const int64_t* budgets, int32_t Hkv, int64_t L, in
   return SGDKV_OK;
 }
 
-sgdkv_status from_cuda(cudaError_t e) { return e == cudaSuccess ? SGDKV_OK : SGDKV_ERR_CUDA; }
+thread_local cudaError_t t_last_cuda = cudaSuccess;
+
+sgdkv_status from_cuda(cudaError_t e) {
+  if (e == cudaSuccess) return SGDKV_OK;
+  t_last_cuda = e;
+  return SGDKV_ERR_CUDA;
+}
 
 }  // namespace
 }  // namespace sgdkv
@@ -131,6 +136,8 @@ const char* sgdkv_status_string(int status) {
 int sgdkv_version(void) { return 100; }
 
 uint64_t sgdkv_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+const char* sgdkv_last_cuda_error_string(void) { return cudaGetErrorString(t_last_cuda); }
 
 void sgdkv_debug_set_score_hooks(uint32_t flags, uint64_t wait_ns) {
   g_score_flags = flags;
@@ -206,7 +213,7 @@ sgdkv_status sgdkv_compress_layer(const void* q_win, const void* K, const void* 
   cudaError_t e = launch_score(static_cast<const __nv_bfloat16*>(q_win),
                                static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, pool,
                                pooled, ws, st);
-  if (e != cudaSuccess) return SGDKV_ERR_CUDA;
+  if (e != cudaSuccess) return from_cuda(e);
   return from_cuda(launch_compact(static_cast<const __nv_bfloat16*>(K),
                                   static_cast<const __nv_bfloat16*>(V), pooled, ht, indices_out,
                                   cu_seqlens_out, static_cast<__nv_bfloat16*>(K_out),
@@ -217,14 +224,15 @@ sgdkv_status sgdkv_last_error(void* workspace, void* stream) {
   if (!workspace) return SGDKV_ERR_WORKSPACE;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   uint32_t code = 0;
-  if (cudaMemcpyAsync(&code, workspace, sizeof(code), cudaMemcpyDeviceToHost, st) != cudaSuccess)
-    return SGDKV_ERR_CUDA;
-  if (cudaStreamSynchronize(st) != cudaSuccess) return SGDKV_ERR_CUDA;
+  cudaError_t e;
+  if ((e = cudaMemcpyAsync(&code, workspace, sizeof(code), cudaMemcpyDeviceToHost, st)) != cudaSuccess)
+    return from_cuda(e);
+  if ((e = cudaStreamSynchronize(st)) != cudaSuccess) return from_cuda(e);
   if (code != 0) {
     const uint32_t zero = 0;
-    if (cudaMemcpyAsync(workspace, &zero, sizeof(zero), cudaMemcpyHostToDevice, st) != cudaSuccess)
-      return SGDKV_ERR_CUDA;
-    if (cudaStreamSynchronize(st) != cudaSuccess) return SGDKV_ERR_CUDA;
+    if ((e = cudaMemcpyAsync(workspace, &zero, sizeof(zero), cudaMemcpyHostToDevice, st)) != cudaSuccess)
+      return from_cuda(e);
+    if ((e = cudaStreamSynchronize(st)) != cudaSuccess) return from_cuda(e);
   }
   return static_cast<sgdkv_status>(code);
 }

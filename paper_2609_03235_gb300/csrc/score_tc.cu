@@ -5,22 +5,25 @@
 // window row w seeing keys j <= L - W + w.  With t_rj = (q_r . k_j) * log2(e)/sqrt(d) and
 // the G*W window rows r = g*W + w of KV head h (contiguous in q_win):
 //
-//   pass 1 (score_pass1_tc): D[r][j] = Q_h K_tile^T on the tensor cores (rows on TMEM
-//     lanes, keys on columns); every epilogue thread owns one window row and keeps an
-//     online (max m_r, sum Z_r = sum 2^(t_rj - m_r)) over the keys of its CTA's range;
-//     the per-CTA partials go to the workspace.
+//   pass 1 (score_pass1_tc): D[r][j] = Q_h K_tile^T, window rows on TMEM lanes and keys on
+//     columns (MMA N = 128 keys; row tiles in pairs per TMEM slot).  Every epilogue thread
+//     keeps an online (max m_r, sum Z_r = sum 2^(t_rj - m_r)) for its window rows over its
+//     share of the CTA's keys; the four shares of a row are merged in shared memory and
+//     one partial per CTA goes to the workspace.
 //   pass 2 (score_pass2_tc): merges the partials into lse_r = m_r + log2 Z_r, then
-//     D[j][r] = K_tile Q_h^T (keys on TMEM lanes, rows on columns); every epilogue thread
-//     owns one key and sums 2^(t_rj - lse_r) over the window rows (two warps per key, each
-//     half of the rows, written to two halves of the raw buffer).
-//   pool (maxpool_sum_kernel): scores = max-pool of (raw half 0 + raw half 1).
+//     D[j][r] = K_tile Q_h^T (keys on TMEM lanes, rows on columns, Q_h in shared memory);
+//     every epilogue thread sums 2^(t_rj - lse_r) for its key over a quarter of the window
+//     rows (four warps per key), written to four partial-sum planes of the raw buffer.
+//   pool (maxpool_sum_kernel): scores = max-pool of the sum of the four planes.
 //
-// CTA roles (320 threads): warp 0 lane 0 issues TMA loads (Q once, K tiles of 128 keys
-// through a ring of shared-memory stages); warp 1 allocates the 512 TMEM columns and its
-// lane 0 issues the MMAs; warps 2..9 are the epilogue (two per TMEM lane quarter).  Each
-// CTA owns one KV head and a contiguous range of key tiles.  Every wait on an mbarrier is
-// bounded in time: on expiry the kernel records SGDKV_ERR_TIMEOUT, all roles leave their
-// loops, in-flight copies and MMAs are drained (again bounded) and TMEM is freed.
+// CTA roles (576 threads): warp 0 lane 0 issues TMA loads (Q_h once, K tiles of 128 keys
+// through a ring of shared-memory stages); warp 1 allocates the 512 TMEM columns
+// and its lane 0 issues the MMAs; warps 2..17 are the epilogue (four per TMEM lane
+// quarter).  An epilogue warp loads all its TMEM columns of a slot, releases the slot,
+// then does the arithmetic, so the MMAs of the next slot overlap it.  Each CTA owns one KV
+// head and a contiguous range of key tiles.  Every wait on an mbarrier is bounded in time:
+// on expiry the kernel records SGDKV_ERR_TIMEOUT, all roles leave their loops, in-flight
+// copies and MMAs are drained (again bounded) and TMEM is freed.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -29,14 +32,18 @@
 namespace sgdkv {
 namespace {
 
-constexpr int kThreads = 320;
-constexpr int kEpiWarps = 8;
+constexpr int kThreads = 576;                     // 18 warps
+constexpr int kEpiWarps = 16;
+constexpr int kMaxRegs = 96;   // 18 warps: 5 warps x 96 x 32 fit one 16K-register SM sub-partition
 constexpr int kTileKeys = 128;
 constexpr uint32_t kTmemCols = 512;
 constexpr int kStageBytes = kTileKeys * 256;      // 32 KB: two 128-byte column halves
 constexpr int kHalfBytes = kTileKeys * 128;       // 16 KB
-constexpr int kNumBars = 15;   // kfull[4] kempty[4] tfull[2] tempty[2] qfull drain never
-constexpr int kCtlBytes = 128;                    // barriers + TMEM address + abort flag
+constexpr int kMaxStages = 8;
+constexpr int kNumBars = 2 * kMaxStages + 7;      // kfull kempty tfull[2] tempty[2] qfull drain never
+constexpr int kCtlBytes = 256;                    // barriers + TMEM address + abort flag
+constexpr int kSmemLimit = 232448;                // opt-in dynamic shared memory per CTA
+constexpr int kQBoxRows = 32;                     // TMA box height for Q rows (pass 2)
 constexpr uint32_t kFlagStallMma = 1u;            // test hook: MMA thread waits on `never`
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr uint64_t kDrainNs = 1000000000ull;      // bound on cleanup waits after an abort
@@ -46,10 +53,9 @@ struct TcParams {
   int64_t L;
   int T;          // key tiles (of 128) per head
   int cph;        // CTAs per head
-  int nrt;        // window-row tiles of 128 (pass 1) = ceil(GW / 128)
+  int nrt;        // window-row tiles of 128 = ceil(GW / 128)
   int nstages;    // K ring depth
   int nparts;     // pass 2: partial slots per head written by pass 1
-  int ppc;        // pass 1: partial slots per CTA
   float scale2;   // log2(e) / sqrt(d)
   uint64_t wait_ns;
   uint32_t flags;
@@ -167,7 +173,7 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
       : SGDKV_LD_REGS32(r)
       : "r"(taddr));
 }
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[32]) {
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
       "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
@@ -184,17 +190,54 @@ __device__ __forceinline__ float ex2(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
+// Packed fp32 pairs (sm_100 family f32x2 arithmetic: one instruction for two lanes).
+__device__ __forceinline__ uint64_t pk(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ uint64_t pku(uint32_t lo, uint32_t hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "r"(lo), "r"(hi));
+  return r;
+}
+__device__ __forceinline__ void upk(uint64_t r, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(r));
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+// 2^(v*s - n) for two lanes, accumulated into the packed pair acc.
+__device__ __forceinline__ uint64_t acc_exp2(uint64_t acc, uint32_t v0, uint32_t v1, uint64_t s2,
+                                             uint64_t neg) {
+  float x0, x1;
+  upk(fma2(pku(v0, v1), s2, neg), x0, x1);
+  return add2(acc, pk(ex2(x0), ex2(x1)));
+}
+__device__ __forceinline__ float hsum(uint64_t a, uint64_t b) {
+  float a0, a1, b0, b1;
+  upk(a, a0, a1);
+  upk(b, b0, b1);
+  return (a0 + a1) + (b0 + b1);
+}
 
 // ---------------------------------------------------------------------------------------
 // Shared pieces of both passes
 // ---------------------------------------------------------------------------------------
 struct Smem {
-  uint8_t* q;          // 2 halves x qrows x 128 B
+  uint8_t* q;          // 2 column halves x qrows x 128 B (pass 1: padded to row tiles)
   uint8_t* k;          // nstages x 32 KB
   uint64_t* bars;      // kNumBars
   uint32_t* tmem_slot;
   int* abort_flag;
-  float* tail;         // pass 2: lse2[kMaxRows]
+  float* tail;         // pass 2: -lse2[kMaxRows] (16-byte aligned)
   int qrows;
 };
 
@@ -211,15 +254,15 @@ __device__ __forceinline__ Smem carve(uint8_t* base, int qrows, int nstages) {
   return s;
 }
 __device__ __forceinline__ uint32_t bar_kfull(const Smem& s, int i) { return smem_u32(s.bars + i); }
-__device__ __forceinline__ uint32_t bar_kempty(const Smem& s, int i) { return smem_u32(s.bars + 4 + i); }
-__device__ __forceinline__ uint32_t bar_tfull(const Smem& s, int i) { return smem_u32(s.bars + 8 + i); }
-__device__ __forceinline__ uint32_t bar_tempty(const Smem& s, int i) { return smem_u32(s.bars + 10 + i); }
-__device__ __forceinline__ uint32_t bar_qfull(const Smem& s) { return smem_u32(s.bars + 12); }
-__device__ __forceinline__ uint32_t bar_drain(const Smem& s) { return smem_u32(s.bars + 13); }
-__device__ __forceinline__ uint32_t bar_never(const Smem& s) { return smem_u32(s.bars + 14); }
+__device__ __forceinline__ uint32_t bar_kempty(const Smem& s, int i) { return smem_u32(s.bars + kMaxStages + i); }
+__device__ __forceinline__ uint32_t bar_tfull(const Smem& s, int i) { return smem_u32(s.bars + 2 * kMaxStages + i); }
+__device__ __forceinline__ uint32_t bar_tempty(const Smem& s, int i) { return smem_u32(s.bars + 2 * kMaxStages + 2 + i); }
+__device__ __forceinline__ uint32_t bar_qfull(const Smem& s) { return smem_u32(s.bars + 2 * kMaxStages + 4); }
+__device__ __forceinline__ uint32_t bar_drain(const Smem& s) { return smem_u32(s.bars + 2 * kMaxStages + 5); }
+__device__ __forceinline__ uint32_t bar_never(const Smem& s) { return smem_u32(s.bars + 2 * kMaxStages + 6); }
 
 // Barrier init, TMEM allocation; returns the TMEM base address (all threads).
-__device__ __forceinline__ uint32_t setup(const Smem& s, int nstages) {
+__device__ __forceinline__ uint32_t setup(const Smem& s, int nstages, uint32_t qfull_count) {
   const int warp = threadIdx.x >> 5;
   if (threadIdx.x == 0) {
     for (int i = 0; i < nstages; ++i) {
@@ -230,7 +273,7 @@ __device__ __forceinline__ uint32_t setup(const Smem& s, int nstages) {
       mbar_init(bar_tfull(s, i), 1);
       mbar_init(bar_tempty(s, i), kEpiWarps);
     }
-    mbar_init(bar_qfull(s), 1);
+    mbar_init(bar_qfull(s), qfull_count);
     mbar_init(bar_drain(s), 1);
     mbar_init(bar_never(s), 1);
     *s.abort_flag = 0;
@@ -263,15 +306,18 @@ __device__ __forceinline__ void teardown(uint32_t tmem) {
 
 // TMA producer (one thread): Q rows of head h once, then the CTA's key tiles.
 __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMap* tm_k,
-                        const TcParams& p, int h, int t0, int ntiles, uint32_t* status) {
+                        const TcParams& p, int h, int t0, int ntiles, bool load_q,
+                        uint32_t* status) {
   volatile int* ab = s.abort_flag;
-  const int qboxes = s.qrows / 128;
-  mbar_expect_tx(bar_qfull(s), uint32_t(2 * s.qrows * 128));
-  for (int c = 0; c < 2; ++c)
-    for (int b = 0; b < qboxes; ++b)
-      tma_load_2d(smem_u32(s.q + c * s.qrows * 128 + b * kHalfBytes), tm_q, 64 * c,
-                  h * p.GW + 128 * b, bar_qfull(s));
-  int issued[4] = {0, 0, 0, 0};
+  if (load_q) {
+    mbar_expect_tx(bar_qfull(s), uint32_t(2 * s.qrows * 128));
+    for (int c = 0; c < 2; ++c)
+      for (int b = 0; b < s.qrows / kQBoxRows; ++b)
+        tma_load_2d(smem_u32(s.q + (c * s.qrows + b * kQBoxRows) * 128), tm_q, 64 * c,
+                    h * p.GW + kQBoxRows * b, bar_qfull(s));
+  }
+  int issued[kMaxStages];
+  for (int i = 0; i < kMaxStages; ++i) issued[i] = 0;
   for (int n = 0; n < ntiles; ++n) {
     const int st = n % p.nstages;
     const int use = n / p.nstages;
@@ -286,9 +332,10 @@ __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMa
   if (*ab) {
     // Drain: every copy this thread started must have landed before the CTA exits.
     volatile int no_abort = 0;
-    bwait(bar_qfull(s), 0, &no_abort, kDrainNs, status);
+    if (load_q) bwait(bar_qfull(s), 0, &no_abort, kDrainNs, status);
     for (int st = 0; st < p.nstages; ++st)
-      if (issued[st] > 0) bwait(bar_kfull(s, st), (issued[st] - 1) & 1, &no_abort, kDrainNs, status);
+      if (issued[st] > 0)
+        bwait(bar_kfull(s, st), (issued[st] - 1) & 1, &no_abort, kDrainNs, status);
   }
 }
 
@@ -311,9 +358,53 @@ __device__ void mma_drain(const Smem& s, uint32_t* status) {
 // ---------------------------------------------------------------------------------------
 // Pass 1: per window row, online (max, sum of 2^(t - max)) over the CTA's key range
 // ---------------------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads, 1)
+template <int N>
+__device__ __forceinline__ float chunk_sum(const uint32_t (&v)[N], float s2, float m) {
+  const uint64_t s22 = pk(s2, s2), nm2 = pk(-m, -m);
+  uint64_t a0 = 0, a1 = 0;
+#pragma unroll
+  for (int e = 0; e < N; e += 4) {
+    a0 = acc_exp2(a0, v[e], v[e + 1], s22, nm2);
+    a1 = acc_exp2(a1, v[e + 2], v[e + 3], s22, nm2);
+  }
+  return hsum(a0, a1);
+}
+
+// Folds N logits of one row (raw dot products in v, keys kb .. kb+N-1) into (m, Z), both in
+// log2 units.  Common case: the running max already bounds the chunk to within 2^32, so
+// the chunk is summed against it directly; otherwise (first chunk, a much larger logit,
+// masked lanes) the chunk max is taken first and Z is rescaled.
+template <int N>
+__device__ __forceinline__ void online_fold(uint32_t (&v)[N], int kb, bool edge, int lim,
+                                            float s2, float& m, float& Z) {
+  if (edge) {
+#pragma unroll
+    for (int e = 0; e < N; ++e)
+      if (kb + e > lim) v[e] = 0xff800000u;             // -inf: key not visible to this row
+  }
+  float zc = chunk_sum<N>(v, s2, m);
+  if (!(zc < 4294967296.f)) {
+    float mx = -INFINITY;
+#pragma unroll
+    for (int e = 0; e < N; ++e) mx = fmaxf(mx, __uint_as_float(v[e]));
+    if (mx == -INFINITY) return;
+    const float mn = fmaxf(m, mx * s2);
+    Z = (m == -INFINITY) ? 0.f : Z * ex2(m - mn);
+    m = mn;
+    zc = chunk_sum<N>(v, s2, m);
+  }
+  Z += zc;
+}
+
+// NRT: row tiles of 128 window rows (1..4), taken in groups of two.  Q_h (padded to
+// NRT x 128 rows) sits in shared memory as the MMA's A operand, K tiles are B.  Each
+// (128-key tile, row group) fills one TMEM slot of 256 columns: D[rows][keys] for the
+// group's row tiles side by side, MMA M = 128 rows, N = 128 keys.  The two slots alternate.
+template <int NRT>
+__global__ void __maxnreg__(kMaxRegs)
 score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                TcParams p, Ws ws) {
+  constexpr int NG = (NRT + 1) / 2;            // row groups (slot uses per key tile)
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   if (smem_u32(smem_raw) & 1023u) {
     if (threadIdx.x == 0) record_error(ws.status, SGDKV_ERR_INTERNAL);
@@ -324,17 +415,15 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   const int t0 = int(int64_t(ci) * p.T / p.cph);
   const int t1 = int(int64_t(ci + 1) * p.T / p.cph);
   const int ntiles = t1 - t0;
-  const Smem s = carve(smem_raw, p.nrt * 128, p.nstages);
-  const uint32_t tmem = setup(s, p.nstages);
+  const Smem s = carve(smem_raw, NRT * 128, p.nstages);
+  const uint32_t tmem = setup(s, p.nstages, 1);
   volatile int* ab = s.abort_flag;
-  const int sub = p.nrt >= 3 ? 2 : 1;          // MMA sub-chunks per 128-key tile
-  const int nsub = kTileKeys / sub;            // keys per sub-chunk (MMA N)
 
   if (warp == 0) {
-    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, t0, ntiles, ws.status);
+    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, t0, ntiles, true, ws.status);
   } else if (warp == 1) {
     if (lane == 0) {
-      const uint32_t idesc = idesc_bf16(128, nsub);
+      const uint32_t idesc = idesc_bf16(128, kTileKeys);
       bool ok = mma_start(s, p, ws.status);
       const uint32_t q0 = smem_u32(s.q), qhalf = uint32_t(s.qrows * 128);
       for (int n = 0; ok && n < ntiles; ++n) {
@@ -342,18 +431,20 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
         if (!(ok = bwait(bar_kfull(s, st), (n / p.nstages) & 1, ab, p.wait_ns, ws.status))) break;
         tc_fence_after();
         const uint32_t k0 = smem_u32(s.k + st * kStageBytes);
-        for (int j = 0; j < sub; ++j) {
-          const int u = n * sub + j, slot = u & 1;
+        for (int g = 0; g < NG; ++g) {
+          const int u = n * NG + g, slot = u & 1;
           if (!(ok = bwait(bar_tempty(s, slot), ((u >> 1) & 1) ^ 1, ab, p.wait_ns, ws.status)))
             break;
           tc_fence_after();
-          for (int rt = 0; rt < p.nrt; ++rt)
+          for (int i = 0; i < 2 && 2 * g + i < NRT; ++i) {
+            const int rt = 2 * g + i;
             for (int k = 0; k < 8; ++k) {
               const uint32_t koff = uint32_t((k & 3) * 32), half = uint32_t(k >> 2);
               const uint64_t a = sw128_desc(q0 + half * qhalf + uint32_t(rt) * kHalfBytes + koff);
-              const uint64_t b = sw128_desc(k0 + half * kHalfBytes + uint32_t(j * nsub) * 128 + koff);
-              umma_bf16(tmem + uint32_t(slot * 256 + rt * nsub), a, b, idesc, k > 0 ? 1u : 0u);
+              const uint64_t bd = sw128_desc(k0 + half * kHalfBytes + koff);
+              umma_bf16(tmem + uint32_t(slot * 256 + i * kTileKeys), a, bd, idesc, k > 0 ? 1u : 0u);
             }
+          }
           umma_commit(bar_tfull(s, slot));
         }
         if (ok) umma_commit(bar_kempty(s, st));
@@ -361,71 +452,67 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
       if (!ok) mma_drain(s, ws.status);
     }
   } else {
-    const int ew = warp - 2, q = warp & 3, g = ew >> 2;
-    const bool row_split = p.nrt >= 2;
-    float m[2] = {-INFINITY, -INFINITY}, Z[2] = {0.f, 0.f};
-    const int64_t lim_base = p.L - p.W;
+    // Epilogue: the 4 warps of a TMEM lane quarter q share its 32 rows of every row tile
+    // and split each slot's 128 keys into 4 blocks of 32.
+    const int q = warp & 3, wi = (warp - 2) >> 2;
+    const int lim_base = int(p.L - p.W);       // Hkv * L < 2^31
+    float m[NRT], Z[NRT];
+    int lim[NRT];
+    bool valid[NRT];
+#pragma unroll
+    for (int rt = 0; rt < NRT; ++rt) {
+      m[rt] = -INFINITY;
+      Z[rt] = 0.f;
+      valid[rt] = rt * 128 + 32 * q < p.GW;                  // warp-uniform
+      lim[rt] = lim_base + (rt * 128 + 32 * q + lane) % p.W;
+    }
     bool ok = true;
     for (int n = 0; ok && n < ntiles; ++n) {
-      const int64_t key0 = int64_t(t0 + n) * kTileKeys;
-      for (int j = 0; j < sub; ++j) {
-        const int u = n * sub + j, slot = u & 1;
+      const int kb = (t0 + n) * kTileKeys + wi * 32;
+      const bool edge = kb + 31 > lim_base;
+#pragma unroll
+      for (int g = 0; g < NG; ++g) {
+        const int u = n * NG + g, slot = u & 1;
         if (!(ok = bwait(bar_tfull(s, slot), (u >> 1) & 1, ab, p.wait_ns, ws.status))) break;
         tc_fence_after();
+        uint32_t v[2][32];
+        const uint32_t tb = tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256 + wi * 32);
 #pragma unroll
-        for (int i = 0; i < 2; ++i) {
-          const int rt = row_split ? g + 2 * i : 0;
-          const int r0 = rt * 128 + 32 * q;
-          // warp-uniform: row tile present and not padding
-          if (rt >= p.nrt || (!row_split && i > 0) || r0 >= p.GW) continue;
-          const int64_t lim = lim_base + (r0 + lane) % p.W;
-          const int c_lo = row_split ? 0 : g * (nsub / 2);
-          const int c_hi = row_split ? nsub : c_lo + nsub / 2;
-          for (int c0 = c_lo; c0 < c_hi; c0 += 32) {
-            uint32_t v[32];
-            tmem_ld32(tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256 + rt * nsub + c0), v);
-            tmem_wait_ld();
-            const int64_t kb = key0 + j * nsub + c0;
-            float x[32];
-            float mx = -INFINITY;
-            if (kb + 31 > lim_base) {
-#pragma unroll
-              for (int e = 0; e < 32; ++e) {
-                x[e] = (kb + e <= lim) ? __uint_as_float(v[e]) : -INFINITY;
-                mx = fmaxf(mx, x[e]);
-              }
-            } else {
-#pragma unroll
-              for (int e = 0; e < 32; ++e) {
-                x[e] = __uint_as_float(v[e]);
-                mx = fmaxf(mx, x[e]);
-              }
-            }
-            if (mx == -INFINITY) continue;
-            const float mn = fmaxf(m[i], mx * p.scale2);
-            if (mn > m[i]) {
-              Z[i] = (m[i] == -INFINITY) ? 0.f : Z[i] * ex2(m[i] - mn);
-              m[i] = mn;
-            }
-            float zc = 0.f;
-#pragma unroll
-            for (int e = 0; e < 32; ++e) zc += ex2(fmaf(x[e], p.scale2, -m[i]));
-            Z[i] += zc;
-          }
-        }
+        for (int i = 0; i < 2; ++i)
+          if (2 * g + i < NRT && valid[2 * g + i]) tmem_ld32(tb + uint32_t(i * kTileKeys), v[i]);
+        tmem_wait_ld();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(bar_tempty(s, slot));
+        if (lane == 0) mbar_arrive(bar_tempty(s, slot));   // slot free: data is in registers
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+          const int rt = 2 * g + i;
+          if (rt < NRT && valid[rt]) online_fold<32>(v[i], kb, edge, lim[rt], p.scale2, m[rt], Z[rt]);
+        }
       }
     }
-    if (ok) {
-      const int slot_base = ci * p.ppc + (row_split ? 0 : g);
+    // Merge the 4 key shares of every row in shared memory (the K ring is idle by now: all
+    // tiles were consumed) and write one partial per row per CTA.
+    float2* red = reinterpret_cast<float2*>(s.k);           // [4][kMaxRows]
 #pragma unroll
-      for (int i = 0; i < 2; ++i) {
-        const int rt = row_split ? g + 2 * i : 0;
+    for (int rt = 0; rt < NRT; ++rt)
+      if (valid[rt]) red[wi * kMaxRows + rt * 128 + 32 * q + lane] = make_float2(m[rt], Z[rt]);
+    asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+    if (wi == 0 && !*ab) {
+#pragma unroll
+      for (int rt = 0; rt < NRT; ++rt) {
+        if (!valid[rt]) continue;
         const int r = rt * 128 + 32 * q + lane;
-        if (rt >= p.nrt || (!row_split && i > 0) || rt * 128 + 32 * q >= p.GW) continue;
-        ws.partial[(int64_t(h) * kMaxScoreParts + slot_base) * kMaxRows + r] = make_float2(m[i], Z[i]);
+        float M = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) M = fmaxf(M, red[i * kMaxRows + r].x);
+        float S = 0.f;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float2 e = red[i * kMaxRows + r];
+          if (e.x != -INFINITY) S += e.y * ex2(e.x - M);
+        }
+        ws.partial[(int64_t(h) * kMaxScoreParts + ci) * kMaxRows + r] = make_float2(M, S);
       }
     }
   }
@@ -435,7 +522,7 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
 // ---------------------------------------------------------------------------------------
 // Pass 2: per key, sum over window rows of 2^(t - lse)
 // ---------------------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __maxnreg__(kMaxRegs)
 score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                TcParams p, Ws ws) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -448,15 +535,15 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   const int t0 = int(int64_t(ci) * p.T / p.cph);
   const int t1 = int(int64_t(ci + 1) * p.T / p.cph);
   const int ntiles = t1 - t0;
-  const Smem s = carve(smem_raw, p.nrt * 128, p.nstages);
-  float* lse2 = s.tail;                          // [kMaxRows]
-  const uint32_t tmem = setup(s, p.nstages);
+  const Smem s = carve(smem_raw, p.GW, p.nstages);
+  float* lse2 = s.tail;                          // [kMaxRows], negated
+  const uint32_t tmem = setup(s, p.nstages, 1);
   volatile int* ab = s.abort_flag;
   const int nch = p.GW > 256 ? 2 : 1;            // N chunks of the window rows per tile
   const int nn = p.GW / nch;                     // MMA N
 
   if (warp == 0) {
-    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, t0, ntiles, ws.status);
+    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, t0, ntiles, true, ws.status);
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(128, nn);
@@ -485,7 +572,7 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
       if (!ok) mma_drain(s, ws.status);
     }
   } else {
-    const int ew = warp - 2, q = warp & 3, g = ew >> 2;
+    const int ew = warp - 2, q = warp & 3, wi = ew >> 2;
     // Merge pass-1 partials of every window row into lse2 (log2 units).
     for (int r = ew * 32 + lane; r < p.GW; r += kEpiWarps * 32) {
       const float2* pp = ws.partial + int64_t(h) * kMaxScoreParts * kMaxRows + r;
@@ -496,75 +583,72 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
         const float2 v = pp[int64_t(i) * kMaxRows];
         if (v.x != -INFINITY) S += v.y * ex2(v.x - M);
       }
-      lse2[r] = M + log2f(S);
+      lse2[r] = -(M + log2f(S));                  // stored negated: the bias of the FMA
     }
     asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
-    // columns of each N chunk handled by this warp group: split at a multiple of 16
-    const int split = ((nn / 2 + 15) / 16) * 16;
-    const int c_lo = g ? split : 0;
-    const int half_cols = g ? nn - split : split;
-    float* raw_out = ws.raw + int64_t(g) * p.Hkv * p.L + int64_t(h) * p.L;
-    const int64_t lim_base = p.L - p.W;
+    const uint64_t s22 = pk(p.scale2, p.scale2);
+    // The 4 warps of lane quarter q share its 32 keys; the window rows of every N chunk
+    // are dealt to them in blocks of 16 columns, round robin over the whole tile.
+    const int gpc = nn / 16;                     // 16-column blocks per chunk (<= 16)
+    float* raw_out = ws.raw + int64_t(wi) * p.Hkv * p.L + int64_t(h) * p.L;
+    const int lim_base = int(p.L - p.W);
     bool ok = true;
     for (int n = 0; ok && n < ntiles; ++n) {
-      const int64_t key0 = int64_t(t0 + n) * kTileKeys;
-      const int64_t j = key0 + 32 * q + lane;
+      const int key0 = (t0 + n) * kTileKeys;
+      const int j = key0 + 32 * q + lane;
       const bool masked = key0 + kTileKeys - 1 > lim_base;
-      float acc = 0.f;
+      uint64_t acc0 = 0, acc1 = 0;
       for (int c = 0; c < nch; ++c) {
         const int u = n * nch + c, slot = u & 1;
         if (!(ok = bwait(bar_tfull(s, slot), (u >> 1) & 1, ab, p.wait_ns, ws.status))) break;
         tc_fence_after();
-        const uint32_t tbase = tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256);
-        for (int c0 = 0; c0 < half_cols; c0 += 32) {
-          uint32_t v[32];
-          const bool full = c0 + 32 <= half_cols;
-          if (full) tmem_ld32(tbase + uint32_t(c_lo + c0), v);
-          else tmem_ld16(tbase + uint32_t(c_lo + c0), v);
-          tmem_wait_ld();
-          const int nv = full ? 32 : 16;
-          const int rbase = c * nn + c_lo + c0;
-          if (!masked) {
-            if (full) {
+        const int li0 = (((wi - c * gpc) % 4) + 4) % 4;   // first block of this warp in chunk c
+        const int ng = li0 < gpc ? (gpc - li0 + 3) / 4 : 0;
+        const uint32_t tb = tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256);
+        uint32_t v[4][16];
 #pragma unroll
-              for (int e = 0; e < 32; ++e)
-                acc += ex2(fmaf(__uint_as_float(v[e]), p.scale2, -lse2[rbase + e]));
-            } else {
-#pragma unroll
-              for (int e = 0; e < 16; ++e)
-                acc += ex2(fmaf(__uint_as_float(v[e]), p.scale2, -lse2[rbase + e]));
-            }
-          } else {
-#pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              const int r = rbase + e;
-              if (e < nv && j <= lim_base + r % p.W)
-                acc += ex2(fmaf(__uint_as_float(v[e]), p.scale2, -lse2[r]));
-            }
-          }
-        }
+        for (int k = 0; k < 4; ++k)
+          if (k < ng) tmem_ld16(tb + uint32_t((li0 + 4 * k) * 16), v[k]);
+        tmem_wait_ld();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(bar_tempty(s, slot));
+        if (lane == 0) mbar_arrive(bar_tempty(s, slot));   // slot free: data is in registers
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          if (k >= ng) continue;
+          const int r0 = c * nn + (li0 + 4 * k) * 16;
+          if (masked) {                            // rows that cannot see key j drop out
+#pragma unroll
+            for (int e = 0; e < 16; ++e)
+              if (j > lim_base + (r0 + e) % p.W) v[k][e] = 0xff800000u;
+          }
+          const float4* nl = reinterpret_cast<const float4*>(lse2 + r0);
+#pragma unroll
+          for (int e = 0; e < 16; e += 4) {
+            const float4 b = nl[e >> 2];
+            acc0 = acc_exp2(acc0, v[k][e], v[k][e + 1], s22, pk(b.x, b.y));
+            acc1 = acc_exp2(acc1, v[k][e + 2], v[k][e + 3], s22, pk(b.z, b.w));
+          }
+        }
       }
-      if (ok && j < p.L) raw_out[j] = acc;
+      if (ok && j < p.L) raw_out[j] = hsum(acc0, acc1);
     }
   }
   teardown(tmem);
 }
 
-// scores = max-pool over [j - radius, j + radius] (clipped) of raw0 + raw1.
+// scores = max-pool over [j - radius, j + radius] (clipped) of the four partial sums.
 __global__ void maxpool_sum_kernel(const float* __restrict__ raw, float* __restrict__ out,
                                    int64_t L, int64_t n, int radius) {
   const int64_t t = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
   if (t >= n) return;
   const int64_t j = t % L;
   const float* r0 = raw + (t - j);
-  const float* r1 = r0 + n;
-  float m = r0[j] + r1[j];
+  auto at = [&](int64_t i) { return (r0[i] + r0[n + i]) + (r0[2 * n + i] + r0[3 * n + i]); };
+  float m = at(j);
   for (int s = 1; s <= radius; ++s) {
-    if (j - s >= 0) m = fmaxf(m, r0[j - s] + r1[j - s]);
-    if (j + s < L) m = fmaxf(m, r0[j + s] + r1[j + s]);
+    if (j - s >= 0) m = fmaxf(m, at(j - s));
+    if (j + s < L) m = fmaxf(m, at(j + s));
   }
   out[t] = m;
 }
@@ -585,13 +669,13 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// 2-D bf16 map over a [rows][128] row-major matrix, box {64 columns, 128 rows}, 128B swizzle.
-bool make_map(CUtensorMap* map, const void* base, uint64_t rows) {
+// 2-D bf16 map over a [rows][128] row-major matrix, box {64 columns, box_rows}, 128B swizzle.
+bool make_map(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows) {
   auto fn = encode_fn();
   if (!fn) return false;
   const cuuint64_t dims[2] = {cuuint64_t(kD), cuuint64_t(rows)};
   const cuuint64_t strides[1] = {cuuint64_t(kD * 2)};
-  const cuuint32_t box[2] = {64, 128};
+  const cuuint32_t box[2] = {64, box_rows};
   const cuuint32_t estr[2] = {1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -625,30 +709,42 @@ cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq,
   if (p.cph < 1) p.cph = 1;
   if (p.cph > p.T) p.cph = p.T;
   p.nrt = int(ceil_div(p.GW, 128));
-  p.nstages = p.GW > 256 ? 2 : 4;
-  p.ppc = p.nrt >= 2 ? 1 : 2;
-  p.nparts = p.cph * p.ppc;
+  p.nparts = p.cph;
   if (p.nparts > kMaxScoreParts) return cudaErrorInvalidConfiguration;
   p.scale2 = kLog2e / sqrtf(float(kD));
   p.wait_ns = g_score_wait_ns;
   p.flags = g_score_flags;
 
   CUtensorMap tm_q, tm_k;
-  if (!make_map(&tm_q, q, uint64_t(Hq) * W) || !make_map(&tm_k, K, uint64_t(Hkv) * L))
+  if (!make_map(&tm_q, q, uint64_t(Hq) * W, kQBoxRows) ||
+      !make_map(&tm_k, K, uint64_t(Hkv) * L, kTileKeys))
     return cudaErrorInvalidValue;
-  const size_t base = size_t(2) * p.nrt * 128 * 128 + size_t(p.nstages) * kStageBytes + kCtlBytes;
-  const size_t smem1 = base;
-  const size_t smem2 = base + kMaxRows * sizeof(float);
+  // K ring depth: as many 32 KB stages as fit next to each pass's other shared data.
+  TcParams p1 = p, p2 = p;
+  const size_t fixed1 = size_t(2) * p.nrt * 128 * 128 + kCtlBytes;   // Q padded to row tiles
+  const size_t fixed2 = size_t(2) * p.GW * 128 + kCtlBytes + kMaxRows * sizeof(float);
+  p1.nstages = int((kSmemLimit - fixed1) / kStageBytes);
+  p2.nstages = int((kSmemLimit - fixed2) / kStageBytes);
+  if (p1.nstages > kMaxStages) p1.nstages = kMaxStages;
+  if (p2.nstages > kMaxStages) p2.nstages = kMaxStages;
+  if (p1.nstages < 2 || p2.nstages < 2) return cudaErrorInvalidConfiguration;
+  const size_t smem1 = fixed1 + size_t(p1.nstages) * kStageBytes;
+  const size_t smem2 = fixed2 + size_t(p2.nstages) * kStageBytes;
+  // the pass-1 row-merge buffer reuses the K ring once it is idle
+  static_assert(4 * kMaxRows * sizeof(float2) <= size_t(2) * kStageBytes, "merge buffer");
+  void (*pass1)(const CUtensorMap, const CUtensorMap, TcParams, Ws) =
+      p.nrt == 1 ? score_pass1_tc<1>
+                 : (p.nrt == 2 ? score_pass1_tc<2> : (p.nrt == 3 ? score_pass1_tc<3> : score_pass1_tc<4>));
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(score_pass1_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if ((e = cudaFuncSetAttribute(pass1, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 int(smem1))) != cudaSuccess)
     return e;
   if ((e = cudaFuncSetAttribute(score_pass2_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 int(smem2))) != cudaSuccess)
     return e;
   const int grid = Hkv * p.cph;
-  score_pass1_tc<<<grid, kThreads, smem1, stream>>>(tm_q, tm_k, p, ws);
-  score_pass2_tc<<<grid, kThreads, smem2, stream>>>(tm_q, tm_k, p, ws);
+  pass1<<<grid, kThreads, smem1, stream>>>(tm_q, tm_k, p1, ws);
+  score_pass2_tc<<<grid, kThreads, smem2, stream>>>(tm_q, tm_k, p2, ws);
   const int64_t n = int64_t(Hkv) * L;
   maxpool_sum_kernel<<<unsigned(ceil_div(n, 256)), 256, 0, stream>>>(ws.raw, scores_out, L, n,
                                                                     pool / 2);

@@ -4,9 +4,9 @@
 //
 // Scores are finite and non-negative, so their fp32 bit patterns sort like their values
 // and the threshold search is an exact most-significant-digit radix select on uint32 keys:
-// four 8-bit passes, each a histogram over the keys that match the digits fixed so far.
-// The CTA that finishes a pass last (atomic completion counter, no waiting) picks the next
-// digit.  Compaction then keeps every middle key above the threshold tau plus the first
+// four passes of 8-bit digits, each a histogram over the keys that match the digits fixed
+// so far.  The CTA that finishes a pass last (atomic completion counter,
+// no waiting) picks the next digit and clears the histogram for the next pass or call.  Compaction then keeps every middle key above the threshold tau plus the first
 // `tie_quota` keys equal to tau in position order, and writes kept positions ascending.
 #include "sgdkv_internal.cuh"
 
@@ -43,34 +43,23 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* s_warp
   return r;
 }
 
-// Reset the per-head selection state and write cu_seqlens.
-__global__ void sel_init_kernel(HeadTable ht, Ws ws, int32_t* cu_out) {
-  const int h = blockIdx.x;
-  for (int i = threadIdx.x; i < 256; i += blockDim.x) ws.hist[h * 256 + i] = 0u;
-  if (threadIdx.x == 0) {
-    SelState s{};
-    s.prefix = 0u;
-    s.k_rem = uint32_t(ht.k_mid[h]);
-    s.tau = 0u;
-    s.tie_quota = 0u;
-    ws.sel[h] = s;
-    ws.sel_cnt[h] = 0u;
-    cu_out[h] = ht.cu[h];
-    if (h == ht.Hkv - 1) cu_out[h + 1] = ht.cu[h + 1];
-  }
-}
-
-// One 8-bit digit of the radix select over the middle range of every head.
+// One 8-bit digit (bits 24-31, 16-23, 8-15, 0-7 in passes 0..3) of the radix select over
+// the middle range of every head.  Each warp counts into its own shared-memory histogram
+// (neighbouring positions have similar scores, so lanes of a warp often share a bin; the
+// contention stays inside the warp), then the CTA adds its counts to the head's global
+// histogram.
 __global__ void __launch_bounds__(kSelThreads)
 sel_radix_kernel(const float* __restrict__ scores, HeadTable ht, Ws ws, int pass, int nchunks) {
-  const int h = blockIdx.y, c = blockIdx.x, tid = threadIdx.x;
+  constexpr int kWarps = kSelThreads / 32;
+  const int h = blockIdx.y, c = blockIdx.x, tid = threadIdx.x, wid = tid >> 5;
   if (ht.k_mid[h] == 0) return;   // nothing to select from the middle of this head
-  __shared__ uint32_t hist[256];
+  __shared__ uint32_t hist[kWarps][kRadixBins];
+  __shared__ uint32_t s_warp[kWarps + 1];
   __shared__ int s_last;
-  for (int i = tid; i < 256; i += blockDim.x) hist[i] = 0u;
+  for (int i = tid; i < kWarps * kRadixBins; i += blockDim.x) (&hist[0][0])[i] = 0u;
   __syncthreads();
-  const uint32_t prefix = ws.sel[h].prefix;
   const int shift = 24 - 8 * pass;
+  const uint32_t prefix = pass == 0 ? 0u : ws.sel[h].prefix;
   const uint32_t hi_mask = pass == 0 ? 0u : (0xffffffffu << (32 - 8 * pass));
   const int64_t L = ht.L, mid_lo = ht.n_sink, mid_hi = ht.L - ht.n_recent;
   const int64_t beg = mid_lo + int64_t(c) * kSelChunk;
@@ -78,55 +67,37 @@ sel_radix_kernel(const float* __restrict__ scores, HeadTable ht, Ws ws, int pass
   const float* row = scores + int64_t(h) * L;
   for (int64_t j = beg + tid; j < end; j += blockDim.x) {
     const uint32_t u = __float_as_uint(__ldg(row + j));
-    if ((u & hi_mask) == prefix) atomicAdd(&hist[(u >> shift) & 255u], 1u);
+    if ((u & hi_mask) == prefix) atomicAdd(&hist[wid][(u >> shift) & 255u], 1u);
   }
   __syncthreads();
-  for (int i = tid; i < 256; i += blockDim.x)
-    if (hist[i]) atomicAdd(&ws.hist[h * 256 + i], hist[i]);
+  uint32_t* ghist = ws.hist + int64_t(h) * kRadixBins;
+  {
+    uint32_t cnt = 0;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) cnt += hist[w][tid];
+    if (cnt) atomicAdd(&ghist[tid], cnt);
+  }
   __threadfence();
   __syncthreads();
   if (tid == 0) s_last = (atomicAdd(&ws.sel_cnt[h], 1u) == uint32_t(nchunks - 1));
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  if (tid >= 32) return;
-  // Last CTA of this head: lane l holds bins 255-8l .. 248-8l (descending digit order).
-  const int lane = tid;
-  const uint32_t k_rem = ws.sel[h].k_rem;
-  uint32_t bins[8];
-  uint32_t lsum = 0;
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    bins[i] = __ldcg(&ws.hist[h * 256 + 255 - 8 * lane - i]);
-    lsum += bins[i];
+  // Last CTA of this head: thread t holds bin 255 - t (descending digit order).
+  const uint32_t k_rem = pass == 0 ? uint32_t(ht.k_mid[h]) : ws.sel[h].k_rem;
+  const uint32_t cnt = __ldcg(&ghist[255 - tid]);
+  uint32_t total;
+  const uint32_t excl = block_excl_scan(cnt, s_warp, &total);
+  if (excl < k_rem && excl + cnt >= k_rem) {             // exactly one thread
+    SelState st;
+    st.prefix = prefix | (uint32_t(255 - tid) << shift);
+    st.k_rem = k_rem - excl;
+    st.tau = st.prefix;
+    st.tie_quota = st.k_rem;
+    ws.sel[h] = st;
   }
-  const uint32_t incl = warp_incl_scan(lsum);
-  const uint32_t excl = incl - lsum;
-  const unsigned hit = __ballot_sync(0xffffffffu, incl >= k_rem);
-  const int first = __ffs(hit) - 1;   // k_rem <= total middle count, so some lane hits
-  if (lane == first) {
-    uint32_t cum = excl, digit = 0, rem = k_rem;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      if (cum + bins[i] >= k_rem) {
-        digit = uint32_t(255 - 8 * lane - i);
-        rem = k_rem - cum;
-        break;
-      }
-      cum += bins[i];
-    }
-    SelState s = ws.sel[h];
-    s.prefix = s.prefix | (digit << shift);
-    s.k_rem = rem;
-    if (pass == 3) {
-      s.tau = s.prefix;
-      s.tie_quota = rem;
-    }
-    ws.sel[h] = s;
-  }
-#pragma unroll
-  for (int i = 0; i < 8; ++i) ws.hist[h * 256 + 8 * lane + i] = 0u;
-  if (lane == 0) ws.sel_cnt[h] = 0u;
+  ghist[255 - tid] = 0u;                                   // clear for the next pass / call
+  if (tid == 0) ws.sel_cnt[h] = 0u;
 }
 
 struct KeepRule {
@@ -150,8 +121,13 @@ __device__ __forceinline__ KeepRule keep_rule(const HeadTable& ht, const SelStat
 
 // Per chunk of the whole row: kept tokens that are not ties, and middle ties at tau.
 __global__ void __launch_bounds__(kSelThreads)
-sel_count_kernel(const float* __restrict__ scores, HeadTable ht, Ws ws, int nchunks) {
+sel_count_kernel(const float* __restrict__ scores, HeadTable ht, Ws ws, int nchunks,
+                 int32_t* __restrict__ cu_out) {
   const int h = blockIdx.y, c = blockIdx.x, tid = threadIdx.x;
+  if (c == 0 && tid == 0) {
+    cu_out[h] = ht.cu[h];
+    if (h == ht.Hkv - 1) cu_out[h + 1] = ht.cu[h + 1];
+  }
   const KeepRule kr = keep_rule(ht, ws.sel[h], h);
   const int64_t beg = int64_t(c) * kSelChunk;
   const int64_t end = beg + kSelChunk < kr.L ? beg + kSelChunk : kr.L;
@@ -271,7 +247,6 @@ cudaError_t launch_compact(const __nv_bfloat16* K, const __nv_bfloat16* V,
                            int32_t* cu_out, __nv_bfloat16* K_out, __nv_bfloat16* V_out,
                            int64_t total_rows, const Ws& ws, cudaStream_t stream) {
   const int Hkv = ht.Hkv;
-  sel_init_kernel<<<Hkv, 256, 0, stream>>>(ht, ws, cu_out);
   const int64_t mid = ht.L - ht.n_sink - ht.n_recent;
   const int mid_chunks = int(ceil_div(mid > 0 ? mid : 1, kSelChunk));
   for (int pass = 0; pass < 4; ++pass)
@@ -279,10 +254,10 @@ cudaError_t launch_compact(const __nv_bfloat16* K, const __nv_bfloat16* V,
                                                                          mid_chunks);
   const int row_chunks = int(ceil_div(ht.L, kSelChunk));
   sel_count_kernel<<<dim3(row_chunks, Hkv), kSelThreads, 0, stream>>>(scores, ht, ws,
-                                                                      row_chunks);
+                                                                      row_chunks, cu_out);
   sel_write_kernel<<<dim3(row_chunks, Hkv), kSelThreads, 0, stream>>>(scores, ht, ws,
                                                                       row_chunks, indices_out);
-  note_launches(7);
+  note_launches(6);
   if (total_rows > 0) {
     note_launches(1);
     int64_t blocks = ceil_div(total_rows * 16, 256);

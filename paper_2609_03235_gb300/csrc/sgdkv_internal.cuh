@@ -17,6 +17,7 @@ constexpr int kMaxScoreParts = 320;    // pass-1 partial (m, Z) slots per KV hea
 constexpr int kSelChunk = 4096;        // selection elements per CTA
 constexpr int kSelThreads = 256;       // threads per selection CTA (16 elements each)
 constexpr int kSelPerThread = kSelChunk / kSelThreads;
+constexpr int kRadixBins = 256;        // radix digit: 8 bits
 
 // Per-head state of the radix selection (lives in the workspace).
 struct SelState {
@@ -38,22 +39,22 @@ struct HeadTable {
   int32_t k_mid[SGDKV_MAX_KV_HEADS];    // middle tokens to select: b_h - n_sink - n_recent
 };
 
-// Device views into the caller's workspace.
+// Device views into the caller's workspace.  The control block (status, histograms,
+// counters, selection state) sits at fixed offsets sized for SGDKV_MAX_KV_HEADS, so the
+// kernels that leave it cleared keep it valid for the next call whatever its shape.
 struct Ws {
   uint32_t* status;      // sticky first device-side error (sgdkv_status)
-  uint32_t* merge_cnt;   // [Hkv] pass-1 completion counters
-  SelState* sel;         // [Hkv]
-  uint32_t* hist;        // [Hkv][256] radix histograms
-  uint32_t* sel_cnt;     // [Hkv] radix-pass completion counters
+  uint32_t* hist;        // [SGDKV_MAX_KV_HEADS][kRadixBins] radix histograms (kept zero)
+  uint32_t* sel_cnt;     // [SGDKV_MAX_KV_HEADS] radix-pass completion counters (kept zero)
+  SelState* sel;         // [SGDKV_MAX_KV_HEADS]
   uint2* chunk_cnt;      // [Hkv][n_sel_chunks] (kept non-ties, ties) per selection chunk
-  float* lse;            // [Hkv][kMaxRows] per window row: log2 of its softmax normaliser
-  float2* partial;       // [Hkv][kMaxScoreParts][kMaxRows] per-part (max, sum) in log2 units
-  float* raw;            // [2][Hkv][L] window scores before pooling, as two partial sums
+  float2* partial;       // [Hkv][kMaxScoreParts][kMaxRows] per-CTA (max, sum), log2 units
+  float* raw;            // [4][Hkv][L] window scores before pooling, as four partial sums
   float* pooled;         // [Hkv][L] pooled scores (compress_layer scratch)
 };
 
 struct WsLayout {
-  size_t status, merge_cnt, sel, hist, sel_cnt, chunk_cnt, lse, partial, raw, pooled, total;
+  size_t status, hist, sel_cnt, sel, chunk_cnt, partial, raw, pooled, total;
 };
 
 inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }

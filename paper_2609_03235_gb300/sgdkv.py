@@ -19,7 +19,8 @@ OK, ERR_INVALID_ARG, ERR_INFEASIBLE_BUDGET, ERR_WORKSPACE, ERR_CUDA, ERR_TIMEOUT
 ALLOC_GREEDY, ALLOC_PROPORTIONAL, ALLOC_THRESHOLD = 0, 1, 2
 EXPORTED = ("sgdkv_status_string", "sgdkv_version", "sgdkv_allocate_budgets",
             "sgdkv_workspace_bytes", "sgdkv_score", "sgdkv_compact", "sgdkv_compress_layer",
-            "sgdkv_last_error", "sgdkv_launch_count", "sgdkv_debug_set_score_hooks")
+            "sgdkv_last_error", "sgdkv_launch_count", "sgdkv_debug_set_score_hooks",
+            "sgdkv_last_cuda_error_string")
 
 
 class LibraryMissing(RuntimeError):
@@ -29,7 +30,10 @@ class LibraryMissing(RuntimeError):
 class SgdkvError(RuntimeError):
     def __init__(self, status: int, where: str):
         self.status = status
-        super().__init__(f"{where}: {status_string(status)} (status {status})")
+        msg = f"{where}: {status_string(status)} (status {status})"
+        if status == ERR_CUDA:
+            msg += ": " + lib().sgdkv_last_cuda_error_string().decode()
+        super().__init__(msg)
 
 
 _lib = None
@@ -62,6 +66,7 @@ def lib():
         L.sgdkv_last_error.restype = ctypes.c_int
         L.sgdkv_last_error.argtypes = [_P, _P]
         L.sgdkv_launch_count.restype = ctypes.c_uint64
+        L.sgdkv_last_cuda_error_string.restype = ctypes.c_char_p
         L.sgdkv_debug_set_score_hooks.restype = None
         L.sgdkv_debug_set_score_hooks.argtypes = [ctypes.c_uint32, ctypes.c_uint64]
         _lib = L
