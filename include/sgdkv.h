@@ -21,9 +21,9 @@
  *     work is enqueued asynchronously on it; host-side argument checks happen before any
  *     launch and leave all outputs untouched on error.
  *   - `workspace` is a device buffer of at least sgdkv_workspace_bytes(...) bytes, 256-byte
- *     aligned, zero-filled once by the caller before its first use.  The library keeps it
- *     in a reusable state after every call.  Calls that share a workspace must be ordered
- *     (same stream or synchronised); calls with separate workspaces may run concurrently.
+ *     aligned, zero-filled once by the caller before its first use (its first word is the
+ *     device status word).  Calls that share a workspace must be ordered (same stream or
+ *     synchronised); calls with separate workspaces may run concurrently.
  *   - Device-side failures (a bounded wait that ran out) are recorded in a status word in
  *     the workspace and reported by sgdkv_last_error.  No call aborts the process, traps,
  *     or falls back to the CPU.

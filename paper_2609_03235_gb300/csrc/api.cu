@@ -26,16 +26,8 @@ WsLayout workspace_layout(int32_t Hkv, int64_t L) {
     off = align256(off + bytes);
     return at;
   };
-  const size_t HM = SGDKV_MAX_KV_HEADS;
   const size_t H = size_t(Hkv);
-  const size_t n_sel_chunks = size_t(ceil_div(L, kSelChunk));
-  // fixed control block
   w.status = take(256);
-  w.hist = take(HM * kRadixBins * sizeof(uint32_t));
-  w.sel_cnt = take(HM * sizeof(uint32_t));
-  w.sel = take(HM * sizeof(SelState));
-  // shape-dependent scratch
-  w.chunk_cnt = take(H * n_sel_chunks * sizeof(uint2));
   w.partial = take(H * size_t(kMaxScoreParts) * kMaxRows * sizeof(float2));
   w.raw = take(4 * H * size_t(L) * sizeof(float));
   w.pooled = take(H * size_t(L) * sizeof(float));
@@ -47,10 +39,6 @@ Ws workspace_view(void* base, const WsLayout& lay) {
   char* b = static_cast<char*>(base);
   Ws ws;
   ws.status = reinterpret_cast<uint32_t*>(b + lay.status);
-  ws.hist = reinterpret_cast<uint32_t*>(b + lay.hist);
-  ws.sel_cnt = reinterpret_cast<uint32_t*>(b + lay.sel_cnt);
-  ws.sel = reinterpret_cast<SelState*>(b + lay.sel);
-  ws.chunk_cnt = reinterpret_cast<uint2*>(b + lay.chunk_cnt);
   ws.partial = reinterpret_cast<float2*>(b + lay.partial);
   ws.raw = reinterpret_cast<float*>(b + lay.raw);
   ws.pooled = reinterpret_cast<float*>(b + lay.pooled);

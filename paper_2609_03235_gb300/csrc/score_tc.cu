@@ -77,14 +77,17 @@ __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
+// The waiting thread is suspended until the phase completes or kSuspendNs elapse, so a
+// waiting warp does not take issue slots from the working warps of its sub-partition.
+constexpr uint32_t kSuspendNs = 20000;
 __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(bar), "r"(parity)
+      : "r"(bar), "r"(parity), "n"(kSuspendNs)
       : "memory");
   return ok != 0;
 }
@@ -102,7 +105,7 @@ __device__ __noinline__ bool bwait(uint32_t bar, uint32_t parity, volatile int* 
   const uint64_t t0 = global_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try(bar, parity)) return true;
-    if ((it & 15u) == 0) {
+    if ((it & 3u) == 0) {
       if (*abort_flag) return false;
       if (global_ns() - t0 > limit_ns) {
         record_error(status, SGDKV_ERR_TIMEOUT);
@@ -573,15 +576,24 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     }
   } else {
     const int ew = warp - 2, q = warp & 3, wi = ew >> 2;
-    // Merge pass-1 partials of every window row into lse2 (log2 units).
+    // Merge pass-1 partials of every window row into lse2 (log2 units): one online pass,
+    // eight independent loads in flight per step.
     for (int r = ew * 32 + lane; r < p.GW; r += kEpiWarps * 32) {
       const float2* pp = ws.partial + int64_t(h) * kMaxScoreParts * kMaxRows + r;
-      float M = -INFINITY;
-      for (int i = 0; i < p.nparts; ++i) M = fmaxf(M, pp[int64_t(i) * kMaxRows].x);
-      float S = 0.f;
-      for (int i = 0; i < p.nparts; ++i) {
-        const float2 v = pp[int64_t(i) * kMaxRows];
-        if (v.x != -INFINITY) S += v.y * ex2(v.x - M);
+      float M = -INFINITY, S = 0.f;
+      for (int i0 = 0; i0 < p.nparts; i0 += 8) {
+        float2 v[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          v[i] = i0 + i < p.nparts ? __ldcg(pp + int64_t(i0 + i) * kMaxRows)
+                                   : make_float2(-INFINITY, 0.f);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          if (v[i].x == -INFINITY) continue;
+          const float mn = fmaxf(M, v[i].x);
+          S = (M == -INFINITY ? 0.f : S * ex2(M - mn)) + v[i].y * ex2(v[i].x - mn);
+          M = mn;
+        }
       }
       lse2[r] = -(M + log2f(S));                  // stored negated: the bias of the FMA
     }

@@ -4,14 +4,38 @@
 //
 // Scores are finite and non-negative, so their fp32 bit patterns sort like their values
 // and the threshold search is an exact most-significant-digit radix select on uint32 keys:
-// four passes of 8-bit digits, each a histogram over the keys that match the digits fixed
-// so far.  The CTA that finishes a pass last (atomic completion counter,
-// no waiting) picks the next digit and clears the histogram for the next pass or call.  Compaction then keeps every middle key above the threshold tau plus the first
-// `tie_quota` keys equal to tau in position order, and writes kept positions ascending.
+// four passes of 8-bit digits, each a histogram over the middle keys that match the digits
+// fixed so far.  One thread-block cluster works on one KV head: every CTA owns a
+// contiguous slice of the row, builds its histogram in shared memory, and after a cluster
+// barrier every CTA sums the cluster's histograms (pushed into its shared memory by its
+// peers through distributed shared memory) and picks the same digit.  The threshold tau and the number of keys equal to tau to keep
+// (lowest positions first) follow.  The same kernel then counts kept positions per slice,
+// exchanges the counts through distributed shared memory, and writes every slice's kept
+// positions, ascending, at their final offsets.  A second kernel copies the kept K/V rows.
+#include <cooperative_groups.h>
+
 #include "sgdkv_internal.cuh"
 
 namespace sgdkv {
+namespace cg = cooperative_groups;
 namespace {
+
+constexpr int kCThreads = 512;                 // threads per selection CTA
+constexpr int kCWarps = kCThreads / 32;
+constexpr int kPer = 8;                        // positions per thread per write round
+constexpr int kRound = kCThreads * kPer;       // positions per write round
+
+constexpr int kMaxCluster = 16;
+
+// Cross-CTA data is pushed: every CTA stores its histogram (and later its counts) into
+// each peer's shared memory, so after the cluster barrier all sums read local memory.
+struct SelShared {
+  uint32_t wh[kCWarps][256];              // per-warp histograms (neighbouring keys share bins)
+  uint32_t hall[2][kMaxCluster][256];     // histograms of every CTA of the cluster, by rank
+  uint32_t call[kMaxCluster][2];          // (kept non-ties, ties) of every CTA, by rank
+  uint32_t s_warp[kCWarps + 1];
+  uint32_t bcast[2];
+};
 
 __device__ __forceinline__ uint32_t warp_incl_scan(uint32_t v) {
   const int lane = threadIdx.x & 31;
@@ -23,7 +47,7 @@ __device__ __forceinline__ uint32_t warp_incl_scan(uint32_t v) {
   return v;
 }
 
-// Exclusive scan of one value per thread over a CTA of kSelThreads threads.
+// Exclusive scan of one value per thread over the CTA; *total gets the CTA sum.
 __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* s_warp,
                                                     uint32_t* total) {
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
@@ -31,164 +55,195 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* s_warp
   if (lane == 31) s_warp[wid] = incl;
   __syncthreads();
   if (wid == 0) {
-    const uint32_t x = lane < kSelThreads / 32 ? s_warp[lane] : 0u;
+    const uint32_t x = lane < kCWarps ? s_warp[lane] : 0u;
     const uint32_t xi = warp_incl_scan(x);
-    if (lane < kSelThreads / 32) s_warp[lane] = xi - x;
-    if (lane == kSelThreads / 32 - 1) s_warp[kSelThreads / 32] = xi;
+    if (lane < kCWarps) s_warp[lane] = xi - x;
+    if (lane == kCWarps - 1) s_warp[kCWarps] = xi;
   }
   __syncthreads();
   const uint32_t r = s_warp[wid] + incl - v;
-  *total = s_warp[kSelThreads / 32];
+  *total = s_warp[kCWarps];
   __syncthreads();
   return r;
 }
 
-// One 8-bit digit (bits 24-31, 16-23, 8-15, 0-7 in passes 0..3) of the radix select over
-// the middle range of every head.  Each warp counts into its own shared-memory histogram
-// (neighbouring positions have similar scores, so lanes of a warp often share a bin; the
-// contention stays inside the warp), then the CTA adds its counts to the head's global
-// histogram.
-__global__ void __launch_bounds__(kSelThreads)
-sel_radix_kernel(const float* __restrict__ scores, HeadTable ht, Ws ws, int pass, int nchunks) {
-  constexpr int kWarps = kSelThreads / 32;
-  const int h = blockIdx.y, c = blockIdx.x, tid = threadIdx.x, wid = tid >> 5;
-  if (ht.k_mid[h] == 0) return;   // nothing to select from the middle of this head
-  __shared__ uint32_t hist[kWarps][kRadixBins];
-  __shared__ uint32_t s_warp[kWarps + 1];
-  __shared__ int s_last;
-  for (int i = tid; i < kWarps * kRadixBins; i += blockDim.x) (&hist[0][0])[i] = 0u;
-  __syncthreads();
-  const int shift = 24 - 8 * pass;
-  const uint32_t prefix = pass == 0 ? 0u : ws.sel[h].prefix;
-  const uint32_t hi_mask = pass == 0 ? 0u : (0xffffffffu << (32 - 8 * pass));
-  const int64_t L = ht.L, mid_lo = ht.n_sink, mid_hi = ht.L - ht.n_recent;
-  const int64_t beg = mid_lo + int64_t(c) * kSelChunk;
-  const int64_t end = beg + kSelChunk < mid_hi ? beg + kSelChunk : mid_hi;
-  const float* row = scores + int64_t(h) * L;
-  for (int64_t j = beg + tid; j < end; j += blockDim.x) {
-    const uint32_t u = __float_as_uint(__ldg(row + j));
-    if ((u & hi_mask) == prefix) atomicAdd(&hist[wid][(u >> shift) & 255u], 1u);
-  }
-  __syncthreads();
-  uint32_t* ghist = ws.hist + int64_t(h) * kRadixBins;
-  {
-    uint32_t cnt = 0;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) cnt += hist[w][tid];
-    if (cnt) atomicAdd(&ghist[tid], cnt);
-  }
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) s_last = (atomicAdd(&ws.sel_cnt[h], 1u) == uint32_t(nchunks - 1));
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  // Last CTA of this head: thread t holds bin 255 - t (descending digit order).
-  const uint32_t k_rem = pass == 0 ? uint32_t(ht.k_mid[h]) : ws.sel[h].k_rem;
-  const uint32_t cnt = __ldcg(&ghist[255 - tid]);
-  uint32_t total;
-  const uint32_t excl = block_excl_scan(cnt, s_warp, &total);
-  if (excl < k_rem && excl + cnt >= k_rem) {             // exactly one thread
-    SelState st;
-    st.prefix = prefix | (uint32_t(255 - tid) << shift);
-    st.k_rem = k_rem - excl;
-    st.tau = st.prefix;
-    st.tie_quota = st.k_rem;
-    ws.sel[h] = st;
-  }
-  ghist[255 - tid] = 0u;                                   // clear for the next pass / call
-  if (tid == 0) ws.sel_cnt[h] = 0u;
-}
-
 struct KeepRule {
-  int64_t L, mid_lo, mid_hi;
+  int64_t mid_lo, mid_hi;
   uint32_t tau;
-  bool none;   // k_mid == 0: keep no middle token
+  bool none;   // nothing selected from the middle
   __device__ __forceinline__ bool protected_pos(int64_t j) const { return j < mid_lo || j >= mid_hi; }
   __device__ __forceinline__ bool above(uint32_t u) const { return !none && u > tau; }
   __device__ __forceinline__ bool tie(uint32_t u) const { return !none && u == tau; }
 };
 
-__device__ __forceinline__ KeepRule keep_rule(const HeadTable& ht, const SelState& s, int h) {
-  KeepRule r;
-  r.L = ht.L;
-  r.mid_lo = ht.n_sink;
-  r.mid_hi = ht.L - ht.n_recent;
-  r.tau = s.tau;
-  r.none = ht.k_mid[h] == 0;
-  return r;
-}
+// One cluster per KV head (grid = Hkv * csize, cluster = csize CTAs).  Control flow is
+// uniform across a cluster, so every CTA reaches every cluster barrier.
+// PER > 0: each thread holds PER consecutive positions of its CTA's slice in registers for
+// the whole kernel (slice <= kCThreads * PER); PER == 0: every pass streams the slice.
+template <int PER>
+__global__ void __launch_bounds__(kCThreads)
+sel_cluster_kernel(const float* __restrict__ scores, HeadTable ht, int csize,
+                   int32_t* __restrict__ indices_out, int32_t* __restrict__ cu_out,
+                   uint32_t* __restrict__ status) {
+  cg::cluster_group cluster = cg::this_cluster();
+  __shared__ SelShared sm;
+  const int tid = threadIdx.x, wid = tid >> 5;
+  const int rank = int(cluster.block_rank());
+  const int h = blockIdx.x / csize;
+  const int64_t L = ht.L;
+  const int64_t slice = ceil_div(L, csize);
+  const int64_t beg = int64_t(rank) * slice < L ? int64_t(rank) * slice : L;
+  const int64_t end = beg + slice < L ? beg + slice : L;
+  const float* row = scores + int64_t(h) * L;
+  KeepRule kr;
+  kr.mid_lo = ht.n_sink;
+  kr.mid_hi = L - ht.n_recent;
+  kr.none = ht.k_mid[h] == 0;
+  const int64_t mb = beg > kr.mid_lo ? beg : kr.mid_lo;     // middle part of this slice
+  const int64_t me = end < kr.mid_hi ? end : kr.mid_hi;
 
-// Per chunk of the whole row: kept tokens that are not ties, and middle ties at tau.
-__global__ void __launch_bounds__(kSelThreads)
-sel_count_kernel(const float* __restrict__ scores, HeadTable ht, Ws ws, int nchunks,
-                 int32_t* __restrict__ cu_out) {
-  const int h = blockIdx.y, c = blockIdx.x, tid = threadIdx.x;
-  if (c == 0 && tid == 0) {
-    cu_out[h] = ht.cu[h];
-    if (h == ht.Hkv - 1) cu_out[h + 1] = ht.cu[h + 1];
+  // register-resident positions p0 .. p0+PER-1 (0 bits outside the slice: never read)
+  const int64_t p0 = beg + int64_t(tid) * (PER > 0 ? PER : 1);
+  uint32_t u[PER > 0 ? PER : 1];
+  if constexpr (PER > 0) {
+#pragma unroll
+    for (int i = 0; i < PER; ++i) u[i] = p0 + i < end ? __float_as_uint(__ldg(row + p0 + i)) : 0u;
   }
-  const KeepRule kr = keep_rule(ht, ws.sel[h], h);
-  const int64_t beg = int64_t(c) * kSelChunk;
-  const int64_t end = beg + kSelChunk < kr.L ? beg + kSelChunk : kr.L;
-  const float* row = scores + int64_t(h) * kr.L;
-  uint32_t nk = 0, nt = 0;
-  for (int64_t j = beg + tid; j < end; j += blockDim.x) {
-    if (kr.protected_pos(j)) {
-      ++nk;
-      continue;
+
+  uint32_t cand = 0u;                       // PER > 0: bit i = position p0+i is middle
+  if constexpr (PER > 0) {
+#pragma unroll
+    for (int i = 0; i < PER; ++i)
+      if (p0 + i >= mb && p0 + i < me) cand |= 1u << i;
+  }
+
+  // ---- radix select of tau over the middle of the row --------------------------------
+  uint32_t prefix = 0u, k_rem = uint32_t(ht.k_mid[h]);
+  if (!kr.none) {
+    for (int pass = 0; pass < 4; ++pass) {
+      const int shift = 24 - 8 * pass;
+      const uint32_t hi_mask = pass == 0 ? 0u : (0xffffffffu << (32 - 8 * pass));
+      for (int i = tid & 31; i < 256; i += 32) sm.wh[wid][i] = 0u;
+      __syncwarp();
+      if constexpr (PER > 0) {
+        // cand: this thread's middle positions still matching the digits fixed so far.
+        // Lanes of a warp that hit the same bin add once (neighbouring positions have
+        // similar scores, so a warp's keys fall into few bins).
+        // A thread's positions are consecutive and pooled scores come in runs, so equal
+        // digits are counted in a register and added once per run.
+        uint32_t keep = 0u, run_bin = 0u, run_len = 0u;
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+          const bool take = ((cand >> i) & 1u) && (u[i] & hi_mask) == prefix;
+          keep |= uint32_t(take) << i;
+          if (take) {
+            const uint32_t d = (u[i] >> shift) & 255u;
+            if (run_len && d != run_bin) {
+              atomicAdd(&sm.wh[wid][run_bin], run_len);
+              run_len = 0u;
+            }
+            run_bin = d;
+            ++run_len;
+          }
+        }
+        if (run_len) atomicAdd(&sm.wh[wid][run_bin], run_len);
+        cand = keep;
+      } else {
+#pragma unroll 4
+        for (int64_t j = mb + tid; j < me; j += kCThreads) {
+          const uint32_t x = __float_as_uint(__ldg(row + j));
+          if ((x & hi_mask) == prefix) atomicAdd(&sm.wh[wid][(x >> shift) & 255u], 1u);
+        }
+      }
+      __syncthreads();
+      if (tid < 256) {
+        uint32_t c = 0;
+#pragma unroll
+        for (int w = 0; w < kCWarps; ++w) c += sm.wh[w][tid];
+        for (int r = 0; r < csize; ++r)     // push to every CTA of the cluster
+          *cluster.map_shared_rank(&sm.hall[pass & 1][rank][tid], r) = c;
+      }
+      cluster.sync();                       // every slice's histogram has arrived
+      // thread t < 256 takes bin 255 - t: descending digit order
+      uint32_t cnt = 0;
+      if (tid < 256)
+        for (int r = 0; r < csize; ++r) cnt += sm.hall[pass & 1][r][255 - tid];
+      uint32_t total;
+      const uint32_t excl = block_excl_scan(cnt, sm.s_warp, &total);
+      if (tid < 256 && excl < k_rem && excl + cnt >= k_rem) {   // exactly one thread
+        sm.bcast[0] = prefix | (uint32_t(255 - tid) << shift);
+        sm.bcast[1] = k_rem - excl;
+      }
+      __syncthreads();
+      prefix = sm.bcast[0];
+      k_rem = sm.bcast[1];
+      // hall[pass & 1] is rewritten two passes later, after the next cluster barrier,
+      // which every CTA reaches only once it has finished reading it.
     }
-    const uint32_t u = __float_as_uint(__ldg(row + j));
-    nk += kr.above(u);
-    nt += kr.tie(u);
   }
-  __shared__ uint32_t s_warp[kSelThreads / 32 + 1];
+  kr.tau = prefix;
+  const uint32_t quota = kr.none ? 0u : k_rem;            // keys equal to tau to keep
+
+  // ---- kept positions per slice, exchanged across the cluster --------------------------
+  uint32_t nk = 0, nt = 0;
+  if constexpr (PER > 0) {
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+      const int64_t j = p0 + i;
+      if (j >= end) continue;
+      if (kr.protected_pos(j)) {
+        ++nk;
+        continue;
+      }
+      nk += kr.above(u[i]);
+      nt += kr.tie(u[i]);
+    }
+  } else {
+    for (int64_t j = beg + tid; j < end; j += kCThreads) {
+      if (kr.protected_pos(j)) {
+        ++nk;
+        continue;
+      }
+      const uint32_t x = __float_as_uint(__ldg(row + j));
+      nk += kr.above(x);
+      nt += kr.tie(x);
+    }
+  }
   uint32_t tot_k, tot_t;
-  block_excl_scan(nk, s_warp, &tot_k);
-  block_excl_scan(nt, s_warp, &tot_t);
-  if (tid == 0) ws.chunk_cnt[int64_t(h) * nchunks + c] = make_uint2(tot_k, tot_t);
-}
-
-// Writes the kept positions of one chunk at their final place in indices_out.
-__global__ void __launch_bounds__(kSelThreads)
-sel_write_kernel(const float* __restrict__ scores, HeadTable ht, Ws ws, int nchunks,
-                 int32_t* __restrict__ indices_out) {
-  const int h = blockIdx.y, c = blockIdx.x, tid = threadIdx.x;
-  const SelState st = ws.sel[h];
-  const KeepRule kr = keep_rule(ht, st, h);
-  __shared__ uint32_t s_warp[kSelThreads / 32 + 1];
-  // Totals of the chunks before this one.
-  uint32_t bk = 0, bt = 0;
-  for (int i = tid; i < c; i += blockDim.x) {
-    const uint2 v = ws.chunk_cnt[int64_t(h) * nchunks + i];
-    bk += v.x;
-    bt += v.y;
+  const uint32_t my_k_before = block_excl_scan(nk, sm.s_warp, &tot_k);
+  const uint32_t my_t_before = block_excl_scan(nt, sm.s_warp, &tot_t);
+  if (tid < csize) {                        // push this slice's counts to CTA `tid`
+    uint32_t* dst = cluster.map_shared_rank(&sm.call[rank][0], tid);
+    dst[0] = tot_k;
+    dst[1] = tot_t;
   }
-  uint32_t before_k, before_t;
-  block_excl_scan(bk, s_warp, &before_k);
-  block_excl_scan(bt, s_warp, &before_t);
-  const uint32_t quota = st.tie_quota;
-  const uint32_t ties_left = before_t < quota ? quota - before_t : 0u;
-  const uint32_t out_base = uint32_t(ht.cu[h]) + before_k + (before_t < quota ? before_t : quota);
-
-  const int64_t beg = int64_t(c) * kSelChunk + int64_t(tid) * kSelPerThread;
-  const float* row = scores + int64_t(h) * kr.L;
-  uint32_t u[kSelPerThread];
-  uint32_t my_ties = 0;
-#pragma unroll
-  for (int i = 0; i < kSelPerThread; ++i) {
-    const int64_t j = beg + i;
-    u[i] = (j < kr.L && !kr.protected_pos(j)) ? __float_as_uint(__ldg(row + j)) : 0u;
-    my_ties += (j < kr.L && !kr.protected_pos(j) && kr.tie(u[i])) ? 1u : 0u;
+  cluster.sync();
+  if (tid == 0) {
+    uint32_t bk = 0, bt = 0;
+    for (int r = 0; r < rank; ++r) {
+      bk += sm.call[r][0];
+      bt += sm.call[r][1];
+    }
+    sm.bcast[0] = bk;
+    sm.bcast[1] = bt;
   }
-  uint32_t dummy;
-  uint32_t tie_rank = block_excl_scan(my_ties, s_warp, &dummy);
-  uint32_t keep_mask = 0, my_keep = 0;
+  __syncthreads();
+  const uint32_t before_k = sm.bcast[0], before_t = sm.bcast[1];
+  uint32_t ties_left = before_t < quota ? quota - before_t : 0u;
+  uint32_t out = uint32_t(ht.cu[h]) + before_k + (before_t < quota ? before_t : quota);
+  const uint32_t out_end = uint32_t(ht.cu[h + 1]);
+
+  if constexpr (PER > 0) {
+    // ---- ordered write from registers (thread order = position order), staged in shared
+    // memory so the copy to indices_out is coalesced ---------------------------------------
+    extern __shared__ int32_t stage[];                  // kCThreads * PER kept positions
+    uint32_t tie_rank = my_t_before;
+    uint32_t slot = my_k_before + (my_t_before < ties_left ? my_t_before : ties_left);
 #pragma unroll
-  for (int i = 0; i < kSelPerThread; ++i) {
-    const int64_t j = beg + i;
-    bool keep = false;
-    if (j < kr.L) {
+    for (int i = 0; i < PER; ++i) {
+      const int64_t j = p0 + i;
+      if (j >= end) continue;
+      bool keep;
       if (kr.protected_pos(j)) {
         keep = true;
       } else if (kr.above(u[i])) {
@@ -196,20 +251,71 @@ sel_write_kernel(const float* __restrict__ scores, HeadTable ht, Ws ws, int nchu
       } else if (kr.tie(u[i])) {
         keep = tie_rank < ties_left;
         ++tie_rank;
+      } else {
+        keep = false;
       }
+      if (!keep) continue;
+      if (slot < uint32_t(kCThreads * PER)) stage[slot] = int32_t(j);
+      else record_error(status, SGDKV_ERR_INTERNAL);
+      ++slot;
     }
-    keep_mask |= uint32_t(keep) << i;
-    my_keep += keep;
-  }
-  uint32_t pos = block_excl_scan(my_keep, s_warp, &dummy) + out_base;
-  const uint32_t pos_end = uint32_t(ht.cu[h + 1]);
+    __syncthreads();
+    const uint32_t kept = tot_k + (tot_t < ties_left ? tot_t : ties_left);
+    for (uint32_t i = tid; i < kept && i < uint32_t(kCThreads * PER); i += kCThreads) {
+      if (out + i < out_end) indices_out[out + i] = stage[i];
+      else record_error(status, SGDKV_ERR_INTERNAL);
+    }
+  } else {
+    // ---- ordered write, rounds of kRound positions -------------------------------------
+    for (int64_t r0 = beg; r0 < end; r0 += kRound) {
+      const int64_t q0 = r0 + int64_t(tid) * kPer;
+      uint32_t x[kPer];
+      uint32_t my_ties = 0;
 #pragma unroll
-  for (int i = 0; i < kSelPerThread; ++i) {
-    if (!(keep_mask & (1u << i))) continue;
-    if (pos < pos_end) indices_out[pos] = int32_t(beg + i);
-    else record_error(ws.status, SGDKV_ERR_INTERNAL);
-    ++pos;
+      for (int i = 0; i < kPer; ++i) {
+        const int64_t j = q0 + i;
+        const bool mid = j < end && !kr.protected_pos(j);
+        x[i] = mid ? __float_as_uint(__ldg(row + j)) : 0u;
+        my_ties += (mid && kr.tie(x[i])) ? 1u : 0u;
+      }
+      uint32_t round_ties;
+      uint32_t tie_rank = block_excl_scan(my_ties, sm.s_warp, &round_ties);
+      uint32_t keep_mask = 0, my_keep = 0;
+#pragma unroll
+      for (int i = 0; i < kPer; ++i) {
+        const int64_t j = q0 + i;
+        bool keep = false;
+        if (j < end) {
+          if (kr.protected_pos(j)) {
+            keep = true;
+          } else if (kr.above(x[i])) {
+            keep = true;
+          } else if (kr.tie(x[i])) {
+            keep = tie_rank < ties_left;
+            ++tie_rank;
+          }
+        }
+        keep_mask |= uint32_t(keep) << i;
+        my_keep += keep;
+      }
+      uint32_t round_kept;
+      uint32_t pos = block_excl_scan(my_keep, sm.s_warp, &round_kept) + out;
+#pragma unroll
+      for (int i = 0; i < kPer; ++i) {
+        if (!(keep_mask & (1u << i))) continue;
+        if (pos < out_end) indices_out[pos] = int32_t(q0 + i);
+        else record_error(status, SGDKV_ERR_INTERNAL);
+        ++pos;
+      }
+      out += round_kept;
+      ties_left = round_ties < ties_left ? ties_left - round_ties : 0u;
+    }
   }
+  if (rank == 0 && tid == 0) {
+    cu_out[h] = ht.cu[h];
+    if (h == ht.Hkv - 1) cu_out[h + 1] = ht.cu[h + 1];
+  }
+  cluster.sync();   // no CTA leaves while a peer may still store into its shared memory
 }
 
 // Copies kept rows: 16 threads per 256-byte row of K and of V.
@@ -240,24 +346,82 @@ gather_kernel(const uint4* __restrict__ K, const uint4* __restrict__ V,
   }
 }
 
+// Largest cluster size (16 if the device runs it, else the portable 8) for the selection.
+template <int PER>
+constexpr size_t stage_bytes() { return size_t(kCThreads) * (PER > 0 ? PER : 0) * sizeof(int32_t); }
+
+template <int PER>
+int cluster_size() {
+  static int cached = 0;
+  if (cached == 0) {
+    cached = 8;
+    cudaFuncSetAttribute(sel_cluster_kernel<PER>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         int(stage_bytes<PER>()));
+    if (cudaFuncSetAttribute(sel_cluster_kernel<PER>,
+                             cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(16, 1, 1);
+      cfg.blockDim = dim3(kCThreads, 1, 1);
+      cfg.dynamicSmemBytes = stage_bytes<PER>();
+      cudaLaunchAttribute attr;
+      attr.id = cudaLaunchAttributeClusterDimension;
+      attr.val.clusterDim.x = 16;
+      attr.val.clusterDim.y = 1;
+      attr.val.clusterDim.z = 1;
+      cfg.attrs = &attr;
+      cfg.numAttrs = 1;
+      int n = 0;
+      if (cudaOccupancyMaxPotentialClusterSize(&n, sel_cluster_kernel<PER>, &cfg) ==
+              cudaSuccess &&
+          n >= 16)
+        cached = 16;
+    }
+    cudaGetLastError();   // a refused query leaves the portable size
+  }
+  return cached;
+}
+
+template <int PER>
+cudaError_t launch_select(const float* scores, const HeadTable& ht, int csize,
+                          int32_t* indices_out, int32_t* cu_out, uint32_t* status,
+                          cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(unsigned(ht.Hkv * csize), 1, 1);
+  cfg.blockDim = dim3(kCThreads, 1, 1);
+  cfg.dynamicSmemBytes = stage_bytes<PER>();
+  cfg.stream = stream;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = unsigned(csize);
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, sel_cluster_kernel<PER>, scores, ht, csize, indices_out,
+                            cu_out, status);
+}
+
 }  // namespace
 
 cudaError_t launch_compact(const __nv_bfloat16* K, const __nv_bfloat16* V,
                            const float* scores, const HeadTable& ht, int32_t* indices_out,
                            int32_t* cu_out, __nv_bfloat16* K_out, __nv_bfloat16* V_out,
                            int64_t total_rows, const Ws& ws, cudaStream_t stream) {
-  const int Hkv = ht.Hkv;
-  const int64_t mid = ht.L - ht.n_sink - ht.n_recent;
-  const int mid_chunks = int(ceil_div(mid > 0 ? mid : 1, kSelChunk));
-  for (int pass = 0; pass < 4; ++pass)
-    sel_radix_kernel<<<dim3(mid_chunks, Hkv), kSelThreads, 0, stream>>>(scores, ht, ws, pass,
-                                                                         mid_chunks);
-  const int row_chunks = int(ceil_div(ht.L, kSelChunk));
-  sel_count_kernel<<<dim3(row_chunks, Hkv), kSelThreads, 0, stream>>>(scores, ht, ws,
-                                                                      row_chunks, cu_out);
-  sel_write_kernel<<<dim3(row_chunks, Hkv), kSelThreads, 0, stream>>>(scores, ht, ws,
-                                                                      row_chunks, indices_out);
-  note_launches(6);
+  // slices of up to 32 positions per thread stay in registers for the whole kernel; the
+  // positions per thread follow from the cluster size that kernel actually runs with
+  auto fits = [&](int per, int cs) { return ceil_div(ceil_div(ht.L, cs), kCThreads) <= per; };
+  cudaError_t e;
+  int cs;
+  if (fits(8, cs = cluster_size<8>()))
+    e = launch_select<8>(scores, ht, cs, indices_out, cu_out, ws.status, stream);
+  else if (fits(16, cs = cluster_size<16>()))
+    e = launch_select<16>(scores, ht, cs, indices_out, cu_out, ws.status, stream);
+  else if (fits(32, cs = cluster_size<32>()))
+    e = launch_select<32>(scores, ht, cs, indices_out, cu_out, ws.status, stream);
+  else
+    e = launch_select<0>(scores, ht, cluster_size<0>(), indices_out, cu_out, ws.status, stream);
+  if (e != cudaSuccess) return e;
+  note_launches(1);
   if (total_rows > 0) {
     note_launches(1);
     int64_t blocks = ceil_div(total_rows * 16, 256);

@@ -79,6 +79,7 @@ COMPACT_CASES = [
     (2, 5000, 10, 20, "full"),        # the whole middle selected
     (5, 9000, 100, 28, "random"),     # several selection chunks, ragged tail
     (1, 1, 0, 0, "full"),
+    (2, 200000, 64, 64, "random"),    # several ordered-write rounds per CTA slice
 ]
 
 
