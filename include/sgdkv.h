@@ -119,6 +119,32 @@ SGDKV_API sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq,
                          void* workspace, size_t ws_bytes, void* stream);
 
 /*
+ * sgdkv_score without a workspace argument, for callers that cannot allocate device
+ * memory (for example code running where the allocator is owned by someone else, or a
+ * plugin that may only receive tensors).  No counterpart in the paper: the computation
+ * and the results are those of sgdkv_score with pool, scores_out as there.
+ *
+ * The scratch is a static 64 MiB device array inside this library, held on every GPU that
+ * loads it until the process exits.  Shapes needing more than that (the status word, the
+ * per-CTA row statistics and the four raw-score planes, about 1.3 MiB * Hkv + 16 * Hkv * L
+ * bytes) are rejected with SGDKV_ERR_WORKSPACE before any device work.  The call allocates
+ * nothing: no cudaMalloc, no cudaFree, no allocating library routine.
+ *
+ * status_out: optional device pointer to one uint32; receives the device-side status of
+ *             this call (SGDKV_OK or SGDKV_ERR_TIMEOUT / SGDKV_ERR_INTERNAL), as
+ *             sgdkv_last_error would report it.  NULL skips the copy.
+ * All calls on a device share the one scratch array, which keeps the last call's
+ * contents; the status word is cleared at the start of every call.  Calls that can overlap
+ * on the GPU (different streams, no ordering between them) race on it and give undefined
+ * results.  The first call on each device looks the scratch up (cudaGetSymbolAddress)
+ * with that device current; make that first call before any stream capture.
+ */
+SGDKV_API sgdkv_status sgdkv_score_static(const void* q_win, const void* K, int32_t Hq,
+                                          int32_t Hkv, int64_t L, int32_t d, int32_t W,
+                                          int32_t pool, float* scores_out, uint32_t* status_out,
+                                          void* stream);
+
+/*
  * Token selection and gather (Section 3.3): per KV head keep positions [0, n_sink) and
  * [L - n_recent, L), plus the (b_h - n_sink - n_recent) middle positions with the highest
  * scores (equal scores: lower position first).  Kept positions are written ascending.

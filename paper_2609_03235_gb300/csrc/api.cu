@@ -2,6 +2,7 @@
 #include <atomic>
 #include <cstdint>
 #include <cstring>
+#include <mutex>
 
 #include "sgdkv_internal.cuh"
 
@@ -105,6 +106,37 @@ sgdkv_status from_cuda(cudaError_t e) {
 
 using namespace sgdkv;
 
+// ---------------------------------------------------------------------------------------
+// Scratch for sgdkv_score_static: for callers that cannot allocate device memory
+// themselves.  Lives in this file's module for as long as the library is loaded on a GPU.
+// ---------------------------------------------------------------------------------------
+static constexpr size_t kStaticScratchBytes = size_t(64) << 20;   // 64 MiB per device
+static __device__ __align__(256) uint8_t sgdkv_static_scratch[kStaticScratchBytes];
+
+namespace {
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+void* g_scratch_dev[kMaxDevices] = {};
+
+// Device address of the static scratch on the current device (looked up once per device,
+// with that device current; the host-side name is only a stand-in for it).
+sgdkv_status static_scratch(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return from_cuda(e);
+  if (dev < 0 || dev >= kMaxDevices) return SGDKV_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_dev[dev]) {
+    void* ptr = nullptr;
+    e = cudaGetSymbolAddress(&ptr, sgdkv_static_scratch);
+    if (e != cudaSuccess) return from_cuda(e);
+    g_scratch_dev[dev] = ptr;
+  }
+  *out = g_scratch_dev[dev];
+  return SGDKV_OK;
+}
+}  // namespace
+
 extern "C" {
 
 const char* sgdkv_status_string(int status) {
@@ -150,6 +182,34 @@ sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq, int32_t H
   return from_cuda(launch_score(static_cast<const __nv_bfloat16*>(q_win),
                                 static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, pool,
                                 scores_out, ws, static_cast<cudaStream_t>(stream)));
+}
+
+sgdkv_status sgdkv_score_static(const void* q_win, const void* K, int32_t Hq, int32_t Hkv,
+                                int64_t L, int32_t d, int32_t W, int32_t pool, float* scores_out,
+                                uint32_t* status_out, void* stream) {
+  if (!q_win || !K || !scores_out) return SGDKV_ERR_INVALID_ARG;
+  if (!aligned16(q_win) || !aligned16(K) || !aligned16(scores_out)) return SGDKV_ERR_INVALID_ARG;
+  sgdkv_status s = check_score_shape(Hq, Hkv, L, d, W);
+  if (s != SGDKV_OK) return s;
+  if ((s = check_pool(pool)) != SGDKV_OK) return s;
+  // scoring uses the status word, the pass-1 partials and the raw planes: everything in
+  // the workspace layout before the pooled-score scratch of sgdkv_compress_layer
+  const WsLayout lay = workspace_layout(Hkv, L);
+  if (lay.pooled > kStaticScratchBytes) return SGDKV_ERR_WORKSPACE;
+  void* scratch = nullptr;
+  if ((s = static_scratch(&scratch)) != SGDKV_OK) return s;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const Ws ws = workspace_view(scratch, lay);
+  cudaError_t e = cudaMemsetAsync(ws.status, 0, sizeof(uint32_t), st);   // starts at zero
+  if (e != cudaSuccess) return from_cuda(e);
+  e = launch_score(static_cast<const __nv_bfloat16*>(q_win), static_cast<const __nv_bfloat16*>(K),
+                   Hq, Hkv, L, W, pool, scores_out, ws, st);
+  if (e != cudaSuccess) return from_cuda(e);
+  if (status_out) {
+    e = cudaMemcpyAsync(status_out, ws.status, sizeof(uint32_t), cudaMemcpyDeviceToDevice, st);
+    if (e != cudaSuccess) return from_cuda(e);
+  }
+  return SGDKV_OK;
 }
 
 sgdkv_status sgdkv_compact(const void* K, const void* V, const float* scores,

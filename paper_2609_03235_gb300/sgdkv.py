@@ -20,7 +20,7 @@ ALLOC_GREEDY, ALLOC_PROPORTIONAL, ALLOC_THRESHOLD = 0, 1, 2
 EXPORTED = ("sgdkv_status_string", "sgdkv_version", "sgdkv_allocate_budgets",
             "sgdkv_workspace_bytes", "sgdkv_score", "sgdkv_compact", "sgdkv_compress_layer",
             "sgdkv_last_error", "sgdkv_launch_count", "sgdkv_debug_set_score_hooks",
-            "sgdkv_last_cuda_error_string")
+            "sgdkv_last_cuda_error_string", "sgdkv_score_static")
 
 
 class LibraryMissing(RuntimeError):
@@ -67,6 +67,8 @@ def lib():
         L.sgdkv_last_error.argtypes = [_P, _P]
         L.sgdkv_launch_count.restype = ctypes.c_uint64
         L.sgdkv_last_cuda_error_string.restype = ctypes.c_char_p
+        L.sgdkv_score_static.restype = ctypes.c_int
+        L.sgdkv_score_static.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, _I32, _P, _P, _P]
         L.sgdkv_debug_set_score_hooks.restype = None
         L.sgdkv_debug_set_score_hooks.argtypes = [ctypes.c_uint32, ctypes.c_uint64]
         _lib = L
@@ -127,6 +129,15 @@ def sgdkv_score(q_win, K, W: int, pool: int, scores_out, workspace, stream=None)
     st = lib().sgdkv_score(_ptr(q_win), _ptr(K), Hq, Hkv, L, d, W, pool, _ptr(scores_out),
                            _ptr(workspace), workspace.numel(), _stream(stream))
     _check(st, "sgdkv_score")
+
+
+def sgdkv_score_static(q_win, K, W: int, pool: int, scores_out, status_out=None, stream=None):
+    """sgdkv_score with the library's static scratch instead of a caller workspace."""
+    Hq, _, d = q_win.shape
+    Hkv, L, _ = K.shape
+    st = lib().sgdkv_score_static(_ptr(q_win), _ptr(K), Hq, Hkv, L, d, W, pool,
+                                  _ptr(scores_out), _ptr(status_out), _stream(stream))
+    _check(st, "sgdkv_score_static")
 
 
 def _budgets(b):
