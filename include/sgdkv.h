@@ -189,6 +189,23 @@ SGDKV_API uint64_t sgdkv_launch_count(void);
 SGDKV_API const char* sgdkv_last_cuda_error_string(void);
 
 /*
+ * Diagnostics: per-kernel timing.  While bit k of kind_mask is set, every kernel of kind k
+ * the library launches is bracketed by CUDA events on its launch stream (mask 0 turns timing
+ * off; each bracket adds two event records to the stream).  sgdkv_debug_kernel_timing synchronises
+ * the recorded events of one kernel kind, returns their summed duration in milliseconds and
+ * their count, and forgets them.  No counterpart in the paper; used by the benchmark to
+ * time its dominant kernel inside the timed region.  Errors: INVALID_ARG, CUDA.
+ */
+#define SGDKV_KERNEL_SCORE_PASS1 0   /* window logits, per-row max and sum  */
+#define SGDKV_KERNEL_SCORE_PASS2 1   /* per-key sum of normalised weights   */
+#define SGDKV_KERNEL_POOL 2          /* max-pool of the raw scores          */
+#define SGDKV_KERNEL_SELECT 3        /* threshold select and ordered compaction */
+#define SGDKV_KERNEL_GATHER 4        /* K/V row copy                        */
+#define SGDKV_KERNEL_KINDS 5
+SGDKV_API void sgdkv_debug_enable_kernel_timing(uint32_t kind_mask);
+SGDKV_API sgdkv_status sgdkv_debug_kernel_timing(int kind, double* total_ms, int64_t* launches);
+
+/*
  * Test hook (no counterpart in the paper): sets the time bound, in nanoseconds, of every
  * device-side wait in the scoring kernels (0 restores the default of 2 s), and flags:
  * bit 0 makes the scoring kernels' MMA issuer first wait on a barrier nothing signals, so

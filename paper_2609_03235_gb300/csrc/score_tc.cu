@@ -755,11 +755,20 @@ cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq,
                                 int(smem2))) != cudaSuccess)
     return e;
   const int grid = Hkv * p.cph;
-  pass1<<<grid, kThreads, smem1, stream>>>(tm_q, tm_k, p1, ws);
-  score_pass2_tc<<<grid, kThreads, smem2, stream>>>(tm_q, tm_k, p2, ws);
+  {
+    KernelTimer t(SGDKV_KERNEL_SCORE_PASS1, stream);
+    pass1<<<grid, kThreads, smem1, stream>>>(tm_q, tm_k, p1, ws);
+  }
+  {
+    KernelTimer t(SGDKV_KERNEL_SCORE_PASS2, stream);
+    score_pass2_tc<<<grid, kThreads, smem2, stream>>>(tm_q, tm_k, p2, ws);
+  }
   const int64_t n = int64_t(Hkv) * L;
-  maxpool_sum_kernel<<<unsigned(ceil_div(n, 256)), 256, 0, stream>>>(ws.raw, scores_out, L, n,
-                                                                    pool / 2);
+  {
+    KernelTimer t(SGDKV_KERNEL_POOL, stream);
+    maxpool_sum_kernel<<<unsigned(ceil_div(n, 256)), 256, 0, stream>>>(ws.raw, scores_out, L, n,
+                                                                      pool / 2);
+  }
   note_launches(3);
   return cudaGetLastError();
 }

@@ -411,18 +411,22 @@ cudaError_t launch_compact(const __nv_bfloat16* K, const __nv_bfloat16* V,
   // positions per thread follow from the cluster size that kernel actually runs with
   auto fits = [&](int per, int cs) { return ceil_div(ceil_div(ht.L, cs), kCThreads) <= per; };
   cudaError_t e;
-  int cs;
-  if (fits(8, cs = cluster_size<8>()))
-    e = launch_select<8>(scores, ht, cs, indices_out, cu_out, ws.status, stream);
-  else if (fits(16, cs = cluster_size<16>()))
-    e = launch_select<16>(scores, ht, cs, indices_out, cu_out, ws.status, stream);
-  else if (fits(32, cs = cluster_size<32>()))
-    e = launch_select<32>(scores, ht, cs, indices_out, cu_out, ws.status, stream);
-  else
-    e = launch_select<0>(scores, ht, cluster_size<0>(), indices_out, cu_out, ws.status, stream);
+  {
+    KernelTimer t(SGDKV_KERNEL_SELECT, stream);
+    int cs;
+    if (fits(8, cs = cluster_size<8>()))
+      e = launch_select<8>(scores, ht, cs, indices_out, cu_out, ws.status, stream);
+    else if (fits(16, cs = cluster_size<16>()))
+      e = launch_select<16>(scores, ht, cs, indices_out, cu_out, ws.status, stream);
+    else if (fits(32, cs = cluster_size<32>()))
+      e = launch_select<32>(scores, ht, cs, indices_out, cu_out, ws.status, stream);
+    else
+      e = launch_select<0>(scores, ht, cluster_size<0>(), indices_out, cu_out, ws.status, stream);
+  }
   if (e != cudaSuccess) return e;
   note_launches(1);
   if (total_rows > 0) {
+    KernelTimer tg(SGDKV_KERNEL_GATHER, stream);
     note_launches(1);
     int64_t blocks = ceil_div(total_rows * 16, 256);
     if (blocks > 152 * 16) blocks = 152 * 16;

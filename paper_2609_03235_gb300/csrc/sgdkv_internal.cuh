@@ -49,6 +49,20 @@ __device__ __forceinline__ void record_error(uint32_t* status, uint32_t code) {
 // Counts kernel launches issued by the library (sgdkv_launch_count).
 void note_launches(int n);
 
+// Brackets one kernel launch with CUDA events when kernel timing is enabled.
+class KernelTimer {
+ public:
+  KernelTimer(int kind, cudaStream_t stream);
+  ~KernelTimer();
+  KernelTimer(const KernelTimer&) = delete;
+  KernelTimer& operator=(const KernelTimer&) = delete;
+
+ private:
+  int kind_;
+  cudaStream_t stream_;
+  void* start_ = nullptr;
+};
+
 // Scorer wait bound and test-hook flags (sgdkv_debug_set_score_hooks).
 extern uint64_t g_score_wait_ns;
 extern uint32_t g_score_flags;

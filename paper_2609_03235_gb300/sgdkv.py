@@ -20,7 +20,8 @@ ALLOC_GREEDY, ALLOC_PROPORTIONAL, ALLOC_THRESHOLD = 0, 1, 2
 EXPORTED = ("sgdkv_status_string", "sgdkv_version", "sgdkv_allocate_budgets",
             "sgdkv_workspace_bytes", "sgdkv_score", "sgdkv_compact", "sgdkv_compress_layer",
             "sgdkv_last_error", "sgdkv_launch_count", "sgdkv_debug_set_score_hooks",
-            "sgdkv_last_cuda_error_string", "sgdkv_score_static")
+            "sgdkv_last_cuda_error_string", "sgdkv_score_static",
+            "sgdkv_debug_enable_kernel_timing", "sgdkv_debug_kernel_timing")
 
 
 class LibraryMissing(RuntimeError):
@@ -71,6 +72,11 @@ def lib():
         L.sgdkv_score_static.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, _I32, _P, _P, _P]
         L.sgdkv_debug_set_score_hooks.restype = None
         L.sgdkv_debug_set_score_hooks.argtypes = [ctypes.c_uint32, ctypes.c_uint64]
+        L.sgdkv_debug_enable_kernel_timing.restype = None
+        L.sgdkv_debug_enable_kernel_timing.argtypes = [ctypes.c_uint32]
+        L.sgdkv_debug_kernel_timing.restype = ctypes.c_int
+        L.sgdkv_debug_kernel_timing.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_double),
+                                                ctypes.POINTER(ctypes.c_int64)]
         _lib = L
     return _lib
 
@@ -175,6 +181,26 @@ def sgdkv_launch_count() -> int:
 
 def sgdkv_debug_set_score_hooks(flags: int, wait_ns: int = 0) -> None:
     lib().sgdkv_debug_set_score_hooks(int(flags), int(wait_ns))
+
+
+KERNEL_SCORE_PASS1, KERNEL_SCORE_PASS2, KERNEL_POOL, KERNEL_SELECT, KERNEL_GATHER = range(5)
+
+
+def sgdkv_debug_enable_kernel_timing(kinds=()) -> None:
+    """Times every launch of the given kernel kinds (an empty set turns timing off)."""
+    mask = 0
+    for k in kinds:
+        mask |= 1 << int(k)
+    lib().sgdkv_debug_enable_kernel_timing(mask)
+
+
+def sgdkv_debug_kernel_timing(kind: int):
+    """(summed milliseconds, launches) of the kernels of one kind timed since the last call."""
+    ms, n = ctypes.c_double(0.0), ctypes.c_int64(0)
+    st = lib().sgdkv_debug_kernel_timing(int(kind), ctypes.byref(ms), ctypes.byref(n))
+    if st != OK:
+        raise SgdkvError(st, "sgdkv_debug_kernel_timing")
+    return ms.value, n.value
 
 
 def sgdkv_last_error(workspace, stream=None) -> int:
