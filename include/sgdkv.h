@@ -22,7 +22,8 @@
  *     launch and leave all outputs untouched on error.
  *   - `workspace` is a device buffer of at least sgdkv_workspace_bytes(...) bytes, 256-byte
  *     aligned, zero-filled once by the caller before its first use (its first word is the
- *     device status word).  Calls that share a workspace must be ordered (same stream or
+ *     device status word; it also holds the scorer's key-tile counters, which every call
+ *     leaves at zero).  Calls that share a workspace must be ordered (same stream or
  *     synchronised); calls with separate workspaces may run concurrently.
  *   - Device-side failures (a bounded wait that ran out) are recorded in a status word in
  *     the workspace and reported by sgdkv_last_error.  No call aborts the process, traps,
@@ -134,9 +135,9 @@ SGDKV_API sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq,
  *             this call (SGDKV_OK or SGDKV_ERR_TIMEOUT / SGDKV_ERR_INTERNAL), as
  *             sgdkv_last_error would report it.  NULL skips the copy.
  * All calls on a device share the one scratch array, which keeps the last call's
- * contents; the status word is cleared at the start of every call.  Calls that can overlap
- * on the GPU (different streams, no ordering between them) race on it and give undefined
- * results.  The first call on each device looks the scratch up (cudaGetSymbolAddress)
+ * contents; the status word and the tile counters are cleared at the start of every call.
+ * Calls that can overlap on the GPU (different streams, no ordering between them) race on
+ * it and give undefined results.  The first call on each device looks the scratch up (cudaGetSymbolAddress)
  * with that device current; make that first call before any stream capture.
  */
 SGDKV_API sgdkv_status sgdkv_score_static(const void* q_win, const void* K, int32_t Hq,

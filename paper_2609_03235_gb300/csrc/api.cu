@@ -28,7 +28,7 @@ WsLayout workspace_layout(int32_t Hkv, int64_t L) {
     return at;
   };
   const size_t H = size_t(Hkv);
-  w.status = take(256);
+  w.status = take(kStatusRegionBytes);
   w.partial = take(H * size_t(kMaxScoreParts) * kMaxRows * sizeof(float2));
   w.raw = take(4 * H * size_t(L) * sizeof(float));
   w.pooled = take(H * size_t(L) * sizeof(float));
@@ -40,6 +40,7 @@ Ws workspace_view(void* base, const WsLayout& lay) {
   char* b = static_cast<char*>(base);
   Ws ws;
   ws.status = reinterpret_cast<uint32_t*>(b + lay.status);
+  ws.sched = reinterpret_cast<uint32_t*>(b + lay.status + kSchedOffset);
   ws.partial = reinterpret_cast<float2*>(b + lay.partial);
   ws.raw = reinterpret_cast<float*>(b + lay.raw);
   ws.pooled = reinterpret_cast<float*>(b + lay.pooled);
@@ -200,7 +201,8 @@ sgdkv_status sgdkv_score_static(const void* q_win, const void* K, int32_t Hq, in
   if ((s = static_scratch(&scratch)) != SGDKV_OK) return s;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const Ws ws = workspace_view(scratch, lay);
-  cudaError_t e = cudaMemsetAsync(ws.status, 0, sizeof(uint32_t), st);   // starts at zero
+  // the status word and the scorer's tile counters start at zero
+  cudaError_t e = cudaMemsetAsync(ws.status, 0, kStatusRegionBytes, st);
   if (e != cudaSuccess) return from_cuda(e);
   e = launch_score(static_cast<const __nv_bfloat16*>(q_win), static_cast<const __nv_bfloat16*>(K),
                    Hq, Hkv, L, W, pool, scores_out, ws, st);

@@ -41,7 +41,7 @@ constexpr int kStageBytes = kTileKeys * 256;      // 32 KB: two 128-byte column 
 constexpr int kHalfBytes = kTileKeys * 128;       // 16 KB
 constexpr int kMaxStages = 8;
 constexpr int kNumBars = 2 * kMaxStages + 7;      // kfull kempty tfull[2] tempty[2] qfull drain never
-constexpr int kCtlBytes = 256;                    // barriers + TMEM address + abort flag
+constexpr int kCtlBytes = 256;                    // barriers, TMEM address, abort flag, tile ids
 constexpr int kSmemLimit = 232448;                // opt-in dynamic shared memory per CTA
 constexpr int kQBoxRows = 32;                     // TMA box height for Q rows (pass 2)
 constexpr uint32_t kFlagStallMma = 1u;            // test hook: MMA thread waits on `never`
@@ -52,7 +52,7 @@ struct TcParams {
   int Hkv, G, W, GW;
   int64_t L;
   int T;          // key tiles (of 128) per head
-  int cph;        // CTAs per head
+  int cph;        // CTAs per head (each claims key tiles of its head until none are left)
   int nrt;        // window-row tiles of 128 = ceil(GW / 128)
   int nstages;    // K ring depth
   int nparts;     // pass 2: partial slots per head written by pass 1
@@ -76,6 +76,9 @@ __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
 }
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive2(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0], 2;" ::"r"(bar) : "memory");
 }
 // The waiting thread is suspended until the phase completes or kSuspendNs elapse, so a
 // waiting warp does not take issue slots from the working warps of its sub-partition.
@@ -240,6 +243,8 @@ struct Smem {
   uint64_t* bars;      // kNumBars
   uint32_t* tmem_slot;
   int* abort_flag;
+  volatile int* stile; // [kMaxStages] key tile held by each K stage (-1: no more tiles)
+  volatile int* utile; // [2] key tile whose products fill each TMEM slot (-1: done)
   float* tail;         // pass 2: -lse2[kMaxRows] (16-byte aligned)
   int qrows;
 };
@@ -253,6 +258,8 @@ __device__ __forceinline__ Smem carve(uint8_t* base, int qrows, int nstages) {
   s.bars = reinterpret_cast<uint64_t*>(ctl);
   s.tmem_slot = reinterpret_cast<uint32_t*>(ctl + kNumBars * 8);
   s.abort_flag = reinterpret_cast<int*>(ctl + kNumBars * 8 + 4);
+  s.stile = reinterpret_cast<int*>(ctl + kNumBars * 8 + 8);
+  s.utile = s.stile + kMaxStages;
   s.tail = reinterpret_cast<float*>(ctl + kCtlBytes);
   return s;
 }
@@ -272,8 +279,9 @@ __device__ __forceinline__ uint32_t setup(const Smem& s, int nstages, uint32_t q
       mbar_init(bar_kfull(s, i), 1);
       mbar_init(bar_kempty(s, i), 1);
     }
+    // tfull: one plain arrive of the MMA thread (publishing utile) + its MMA commit
     for (int i = 0; i < 2; ++i) {
-      mbar_init(bar_tfull(s, i), 1);
+      mbar_init(bar_tfull(s, i), 2);
       mbar_init(bar_tempty(s, i), kEpiWarps);
     }
     mbar_init(bar_qfull(s), qfull_count);
@@ -307,9 +315,11 @@ __device__ __forceinline__ void teardown(uint32_t tmem) {
   }
 }
 
-// TMA producer (one thread): Q rows of head h once, then the CTA's key tiles.
+// TMA producer (one thread): Q rows of head h once, then key tiles of head h claimed one
+// at a time from the head's counter (shared by the head's CTAs) until none are left; the
+// stage after the last one carries tile id -1 and no data.
 __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMap* tm_k,
-                        const TcParams& p, int h, int t0, int ntiles, bool load_q,
+                        const TcParams& p, int h, uint32_t* counter, bool load_q,
                         uint32_t* status) {
   volatile int* ab = s.abort_flag;
   if (load_q) {
@@ -321,12 +331,19 @@ __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMa
   }
   int issued[kMaxStages];
   for (int i = 0; i < kMaxStages; ++i) issued[i] = 0;
-  for (int n = 0; n < ntiles; ++n) {
+  for (int n = 0;; ++n) {
     const int st = n % p.nstages;
     const int use = n / p.nstages;
     if (!bwait(bar_kempty(s, st), (use & 1) ^ 1, ab, p.wait_ns, status)) break;
+    const uint32_t tile = atomicAdd(counter, 1u);
+    if (tile >= uint32_t(p.T)) {
+      s.stile[st] = -1;
+      mbar_arrive(bar_kfull(s, st));            // releases the id; no copy in flight
+      break;
+    }
+    s.stile[st] = int(tile);
     mbar_expect_tx(bar_kfull(s, st), kStageBytes);
-    const int row = int(int64_t(h) * p.L + int64_t(t0 + n) * kTileKeys);
+    const int row = int(int64_t(h) * p.L + int64_t(tile) * kTileKeys);
     for (int c = 0; c < 2; ++c)
       tma_load_2d(smem_u32(s.k + st * kStageBytes + c * kHalfBytes), tm_k, 64 * c, row,
                   bar_kfull(s, st));
@@ -348,6 +365,25 @@ __device__ bool mma_start(const Smem& s, const TcParams& p, uint32_t* status) {
   volatile int* ab = s.abort_flag;
   if ((p.flags & kFlagStallMma) && !bwait(bar_never(s), 0, ab, p.wait_ns, status)) return false;
   return bwait(bar_qfull(s), 0, ab, p.wait_ns, status);
+}
+
+// Publishes the key tile of a TMEM slot use to the epilogue (the plain arrive on tfull
+// releases the store; the MMA commit is the barrier's second arrival).  Tile -1 ends the
+// epilogue's loop: both arrivals are made here.
+__device__ __forceinline__ void publish_slot(const Smem& s, int slot, int tile) {
+  s.utile[slot] = tile;
+  if (tile < 0) mbar_arrive2(bar_tfull(s, slot));
+  else mbar_arrive(bar_tfull(s, slot));
+}
+
+// End of a pass, thread 0 after the CTA's last barrier: the head's last CTA to finish resets
+// the head's tile counter (and the finish count) for the next launch.
+__device__ __forceinline__ void finish_claims(uint32_t* counter, uint32_t* finished, int cph) {
+  __threadfence();
+  if (atomicAdd(finished, 1u) == uint32_t(cph - 1)) {
+    atomicExch(counter, 0u);
+    atomicExch(finished, 0u);
+  }
 }
 
 // MMA thread, after an abort: a commit arrives on `drain` once every MMA this thread issued
@@ -415,30 +451,31 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.x / p.cph, ci = blockIdx.x % p.cph;
-  const int t0 = int(int64_t(ci) * p.T / p.cph);
-  const int t1 = int(int64_t(ci + 1) * p.T / p.cph);
-  const int ntiles = t1 - t0;
+  uint32_t* counter = ws.sched + h;
   const Smem s = carve(smem_raw, NRT * 128, p.nstages);
   const uint32_t tmem = setup(s, p.nstages, 1);
   volatile int* ab = s.abort_flag;
 
   if (warp == 0) {
-    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, t0, ntiles, true, ws.status);
+    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, counter, true, ws.status);
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(128, kTileKeys);
       bool ok = mma_start(s, p, ws.status);
       const uint32_t q0 = smem_u32(s.q), qhalf = uint32_t(s.qrows * 128);
-      for (int n = 0; ok && n < ntiles; ++n) {
+      for (int n = 0; ok; ++n) {
         const int st = n % p.nstages;
         if (!(ok = bwait(bar_kfull(s, st), (n / p.nstages) & 1, ab, p.wait_ns, ws.status))) break;
         tc_fence_after();
+        const int tile = s.stile[st];
         const uint32_t k0 = smem_u32(s.k + st * kStageBytes);
         for (int g = 0; g < NG; ++g) {
           const int u = n * NG + g, slot = u & 1;
           if (!(ok = bwait(bar_tempty(s, slot), ((u >> 1) & 1) ^ 1, ab, p.wait_ns, ws.status)))
             break;
           tc_fence_after();
+          publish_slot(s, slot, tile);
+          if (tile < 0) break;
           for (int i = 0; i < 2 && 2 * g + i < NRT; ++i) {
             const int rt = 2 * g + i;
             for (int k = 0; k < 8; ++k) {
@@ -450,6 +487,7 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
           }
           umma_commit(bar_tfull(s, slot));
         }
+        if (tile < 0) break;
         if (ok) umma_commit(bar_kempty(s, st));
       }
       if (!ok) mma_drain(s, ws.status);
@@ -470,14 +508,19 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
       lim[rt] = lim_base + (rt * 128 + 32 * q + lane) % p.W;
     }
     bool ok = true;
-    for (int n = 0; ok && n < ntiles; ++n) {
-      const int kb = (t0 + n) * kTileKeys + wi * 32;
-      const bool edge = kb + 31 > lim_base;
+    for (int n = 0; ok; ++n) {
 #pragma unroll
       for (int g = 0; g < NG; ++g) {
         const int u = n * NG + g, slot = u & 1;
         if (!(ok = bwait(bar_tfull(s, slot), (u >> 1) & 1, ab, p.wait_ns, ws.status))) break;
         tc_fence_after();
+        const int tile = s.utile[slot];
+        if (tile < 0) {
+          ok = false;                              // no more tiles: leave both loops
+          break;
+        }
+        const int kb = tile * kTileKeys + wi * 32;
+        const bool edge = kb + 31 > lim_base;
         uint32_t v[2][32];
         const uint32_t tb = tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256 + wi * 32);
 #pragma unroll
@@ -520,6 +563,7 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     }
   }
   teardown(tmem);
+  if (threadIdx.x == 0) finish_claims(counter, ws.sched + SGDKV_MAX_KV_HEADS + h, p.cph);
 }
 
 // ---------------------------------------------------------------------------------------
@@ -534,10 +578,8 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     return;
   }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int h = blockIdx.x / p.cph, ci = blockIdx.x % p.cph;
-  const int t0 = int(int64_t(ci) * p.T / p.cph);
-  const int t1 = int(int64_t(ci + 1) * p.T / p.cph);
-  const int ntiles = t1 - t0;
+  const int h = blockIdx.x / p.cph;
+  uint32_t* counter = ws.sched + 2 * SGDKV_MAX_KV_HEADS + h;
   const Smem s = carve(smem_raw, p.GW, p.nstages);
   float* lse2 = s.tail;                          // [kMaxRows], negated
   const uint32_t tmem = setup(s, p.nstages, 1);
@@ -546,22 +588,25 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   const int nn = p.GW / nch;                     // MMA N
 
   if (warp == 0) {
-    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, t0, ntiles, true, ws.status);
+    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, counter, true, ws.status);
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(128, nn);
       bool ok = mma_start(s, p, ws.status);
       const uint32_t q0 = smem_u32(s.q), qhalf = uint32_t(s.qrows * 128);
-      for (int n = 0; ok && n < ntiles; ++n) {
+      for (int n = 0; ok; ++n) {
         const int st = n % p.nstages;
         if (!(ok = bwait(bar_kfull(s, st), (n / p.nstages) & 1, ab, p.wait_ns, ws.status))) break;
         tc_fence_after();
+        const int tile = s.stile[st];
         const uint32_t k0 = smem_u32(s.k + st * kStageBytes);
         for (int c = 0; c < nch; ++c) {
           const int u = n * nch + c, slot = u & 1;
           if (!(ok = bwait(bar_tempty(s, slot), ((u >> 1) & 1) ^ 1, ab, p.wait_ns, ws.status)))
             break;
           tc_fence_after();
+          publish_slot(s, slot, tile);
+          if (tile < 0) break;
           for (int k = 0; k < 8; ++k) {
             const uint32_t koff = uint32_t((k & 3) * 32), half = uint32_t(k >> 2);
             const uint64_t a = sw128_desc(k0 + half * kHalfBytes + koff);
@@ -570,6 +615,7 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
           }
           umma_commit(bar_tfull(s, slot));
         }
+        if (tile < 0) break;
         if (ok) umma_commit(bar_kempty(s, st));
       }
       if (!ok) mma_drain(s, ws.status);
@@ -577,18 +623,18 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   } else {
     const int ew = warp - 2, q = warp & 3, wi = ew >> 2;
     // Merge pass-1 partials of every window row into lse2 (log2 units): one online pass,
-    // eight independent loads in flight per step.
+    // sixteen independent loads in flight per step.
     for (int r = ew * 32 + lane; r < p.GW; r += kEpiWarps * 32) {
       const float2* pp = ws.partial + int64_t(h) * kMaxScoreParts * kMaxRows + r;
       float M = -INFINITY, S = 0.f;
-      for (int i0 = 0; i0 < p.nparts; i0 += 8) {
-        float2 v[8];
+      for (int i0 = 0; i0 < p.nparts; i0 += 16) {
+        float2 v[16];
 #pragma unroll
-        for (int i = 0; i < 8; ++i)
+        for (int i = 0; i < 16; ++i)
           v[i] = i0 + i < p.nparts ? __ldcg(pp + int64_t(i0 + i) * kMaxRows)
                                    : make_float2(-INFINITY, 0.f);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
+        for (int i = 0; i < 16; ++i) {
           if (v[i].x == -INFINITY) continue;
           const float mn = fmaxf(M, v[i].x);
           S = (M == -INFINITY ? 0.f : S * ex2(M - mn)) + v[i].y * ex2(v[i].x - mn);
@@ -605,15 +651,21 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     float* raw_out = ws.raw + int64_t(wi) * p.Hkv * p.L + int64_t(h) * p.L;
     const int lim_base = int(p.L - p.W);
     bool ok = true;
-    for (int n = 0; ok && n < ntiles; ++n) {
-      const int key0 = (t0 + n) * kTileKeys;
-      const int j = key0 + 32 * q + lane;
-      const bool masked = key0 + kTileKeys - 1 > lim_base;
+    for (int n = 0; ok; ++n) {
+      int j = 0;
       uint64_t acc0 = 0, acc1 = 0;
       for (int c = 0; c < nch; ++c) {
         const int u = n * nch + c, slot = u & 1;
         if (!(ok = bwait(bar_tfull(s, slot), (u >> 1) & 1, ab, p.wait_ns, ws.status))) break;
         tc_fence_after();
+        const int tile = s.utile[slot];
+        if (tile < 0) {
+          ok = false;                              // no more tiles
+          break;
+        }
+        const int key0 = tile * kTileKeys;
+        j = key0 + 32 * q + lane;
+        const bool masked = key0 + kTileKeys - 1 > lim_base;
         const int li0 = (((wi - c * gpc) % 4) + 4) % 4;   // first block of this warp in chunk c
         const int ng = li0 < gpc ? (gpc - li0 + 3) / 4 : 0;
         const uint32_t tb = tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256);
@@ -647,6 +699,8 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     }
   }
   teardown(tmem);
+  if (threadIdx.x == 0)
+    finish_claims(counter, ws.sched + 3 * SGDKV_MAX_KV_HEADS + h, p.cph);
 }
 
 // scores = max-pool over [j - radius, j + radius] (clipped) of the four partial sums.

@@ -28,14 +28,18 @@ struct HeadTable {
 // Device views into the caller's workspace.
 struct Ws {
   uint32_t* status;      // sticky first device-side error (sgdkv_status)
+  uint32_t* sched;       // [4][SGDKV_MAX_KV_HEADS] key-tile counters and finish counts of
+                         // the two scoring passes (zero between launches)
   float2* partial;       // [Hkv][kMaxScoreParts][kMaxRows] per-CTA (max, sum), log2 units
   float* raw;            // [4][Hkv][L] window scores before pooling, as four partial sums
   float* pooled;         // [Hkv][L] pooled scores (compress_layer scratch)
 };
 
 struct WsLayout {
-  size_t status, partial, raw, pooled, total;
+  size_t status, partial, raw, pooled, total;   // status region: status word, then sched
 };
+constexpr size_t kSchedOffset = 1024;           // byte offset of Ws::sched in the status region
+constexpr size_t kStatusRegionBytes = kSchedOffset + 4 * SGDKV_MAX_KV_HEADS * sizeof(uint32_t);
 
 __host__ __device__ inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 

@@ -194,3 +194,47 @@ def test_rejects_misaligned_pointer(dev):
     with pytest.raises(sg.SgdkvError) as e:
         sg.sgdkv_score(q, K, wl.W, 7, big[1:], ws)
     assert e.value.status == sg.ERR_INVALID_ARG
+
+
+SCHED_BYTES = (1024, 2048)     # the scorer's key-tile counters inside the workspace
+
+
+def test_tile_counters_return_to_zero(dev):
+    """Every scoring pass claims key tiles from per-head counters in the workspace; the
+    last CTA of each head resets them, so the next call (any shape) starts from zero."""
+    for Hq, Hkv, L, W in [(28, 4, 20000, 64), (14, 2, 1000, 32), (8, 8, 640, 32)]:
+        wl = synth.tiny_workload(Hq=Hq, Hkv=Hkv, d=128, L=L, W=W, n_salient=4)
+        inp = synth.tiny_inputs(wl, tag=400 + L)
+        q, K, _ = _upload(inp, dev)
+        ws = sg.make_workspace(Hq, Hkv, L, W, dev)
+        out = torch.empty((Hkv, L), dtype=torch.float32, device=dev)
+        for _ in range(3):
+            sg.sgdkv_score(q, K, W, 7, out, ws)
+        torch.cuda.synchronize()
+        assert sg.sgdkv_last_error(ws) == sg.OK
+        assert int(ws[SCHED_BYTES[0]:SCHED_BYTES[1]].count_nonzero()) == 0
+        exp = O.max_pool(O.window_scores(inp["q"], inp["K"]), 7)
+        assert _within(out.cpu().numpy(), exp).all()
+
+
+def test_layers_on_two_streams(dev):
+    """Two layers scored and compacted at the same time on two streams (one workspace
+    each), as the benchmark overlaps consecutive layers: each matches the oracle."""
+    wl = synth.tiny_workload(Hq=28, Hkv=4, d=128, L=6000, W=64, n_salient=16, floor=256)
+    b = np.array([1500, 700, 2400, 256], np.int64)
+    streams = [torch.cuda.Stream(dev), torch.cuda.Stream(dev)]
+    runs = []
+    for i, s in enumerate(streams):
+        inp = synth.tiny_inputs(wl, tag=500 + i)
+        q, K, V = _upload(inp, dev)
+        ws = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
+        runs.append((inp, q, K, V, ws, s))
+    torch.cuda.synchronize()
+    outs = []
+    for inp, q, K, V, ws, s in runs:
+        with torch.cuda.stream(s):
+            outs.append(sg.compress_layer_alloc(q, K, V, b, wl.W, 7, 128, 128, ws, stream=s))
+    torch.cuda.synchronize()
+    for (inp, q, K, V, ws, s), out in zip(runs, outs):
+        assert sg.sgdkv_last_error(ws) == sg.OK
+        _check_end_to_end(inp, out, b, 128, 128, 7)
