@@ -102,9 +102,8 @@ __device__ __forceinline__ uint64_t global_ns() {
 
 // Waits for the phase of `bar` with the given parity; false if the CTA aborted or the wait
 // ran past limit_ns (then the timeout is recorded and the CTA-wide abort flag raised).
-__device__ __noinline__ bool bwait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                   uint64_t limit_ns, uint32_t* status) {
-  if (mbar_try(bar, parity)) return true;
+__device__ __noinline__ bool bwait_slow(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                        uint64_t limit_ns, uint32_t* status) {
   const uint64_t t0 = global_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try(bar, parity)) return true;
@@ -118,6 +117,19 @@ __device__ __noinline__ bool bwait(uint32_t bar, uint32_t parity, volatile int* 
     }
   }
 }
+// Completed phases (the common case on the critical path) return after one test, inline.
+__device__ __forceinline__ bool bwait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                      uint64_t limit_ns, uint32_t* status) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok ? true : bwait_slow(bar, parity, abort_flag, limit_ns, status);
+}
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
                                             uint32_t bar) {
@@ -128,32 +140,57 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
-// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of 128 bytes in
-// 8-row atoms of 1024 bytes (the layout a TMA box {64 bf16, rows} with SWIZZLE_128B writes).
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-  uint64_t d = 0;
-  d |= uint64_t((saddr >> 4) & 0x3FFFu);
-  d |= uint64_t(1) << 16;              // leading-dimension offset (unused for this layout)
-  d |= uint64_t(1024 >> 4) << 32;      // stride between 8-row groups
-  d |= uint64_t(1) << 46;              // descriptor version
-  d |= uint64_t(2) << 61;              // SWIZZLE_128B
-  return d;
-}
+// Shared-memory matrix descriptor (K-major operand, 128-byte swizzle, rows of 128 bytes in
+// 8-row atoms of 1024 bytes: the layout a TMA box {64 bf16, rows} with SWIZZLE_128B writes),
+// kept as two 32-bit words.  High word: stride between 8-row groups 1024 B, descriptor
+// version 1, SWIZZLE_128B.  Low word: start address / 16 (< 2^14 for shared memory) and the
+// leading-dimension field set to 1 (unused by this layout); an operand advanced by `bytes`
+// has low word + bytes / 16.
+constexpr uint32_t kDescHi = (1024u >> 4) | (1u << 14) | (2u << 29);
+__device__ __forceinline__ uint32_t desc_lo(uint32_t saddr) { return (saddr >> 4) | (1u << 16); }
 // Instruction descriptor, kind::f16: bf16 A and B (K-major), fp32 accumulator, M x N.
 __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(N >> 3) << 17) | (uint32_t(M >> 4) << 24);
 }
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
-                                          uint32_t accumulate) {
+// One lane of the converged warp (the MMA warp runs its loop with all 32 lanes, so the
+// operands stay warp-uniform; the elected lane alone issues MMAs, commits and arrivals).
+__device__ __forceinline__ uint32_t elect_one() {
+  uint32_t e;
   asm volatile(
-      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      "{\n\t.reg .pred P;\n\telect.sync _|P, 0xffffffff;\n\tselp.u32 %0, 1, 0, P;\n\t}"
+      : "=r"(e));
+  return e;
+}
+// tcgen05.mma kind::f16 from low descriptor words, issued by the lane with leader != 0; ACC
+// is a compile-time accumulate flag.
+template <int ACC>
+__device__ __forceinline__ void umma_lo(uint32_t d_tmem, uint32_t a_lo, uint32_t b_lo,
+                                        uint32_t idesc, uint32_t leader) {
+  asm volatile(
+      "{\n\t.reg .b64 ad, bd;\n\t.reg .pred p, l;\n\t"
+      "mov.b64 ad, {%1, %4};\n\tmov.b64 bd, {%2, %4};\n\t"
+      "setp.ne.b32 p, %5, 0;\n\tsetp.ne.b32 l, %6, 0;\n\t"
+      "@l tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_lo), "r"(b_lo), "r"(idesc), "r"(kDescHi), "n"(ACC), "r"(leader)
       : "memory");
 }
-__device__ __forceinline__ void umma_commit(uint32_t bar) {
+// The 8 k steps (16 columns each of the two 64-column halves) of one 128 x N x 128 MMA:
+// A and B advance 32 B per step within a half and jump by their half strides.
+__device__ __forceinline__ void umma_k128(uint32_t d_tmem, uint32_t a_lo, uint32_t a_half,
+                                          uint32_t b_lo, uint32_t b_half, uint32_t idesc,
+                                          uint32_t leader) {
+  umma_lo<0>(d_tmem, a_lo, b_lo, idesc, leader);
+#pragma unroll
+  for (int k = 1; k < 8; ++k) {
+    const uint32_t ka = (k >> 2) * a_half + (k & 3) * 2, kb = (k >> 2) * b_half + (k & 3) * 2;
+    umma_lo<1>(d_tmem, a_lo + ka, b_lo + kb, idesc, leader);
+  }
+}
+__device__ __forceinline__ void umma_commit(uint32_t bar, uint32_t leader) {
   asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      "{\n\t.reg .pred l;\n\tsetp.ne.b32 l, %1, 0;\n\t"
+      "@l tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}" ::"r"(bar),
+      "r"(leader)
       : "memory");
 }
 __device__ __forceinline__ void tc_fence_before() {
@@ -316,8 +353,9 @@ __device__ __forceinline__ void teardown(uint32_t tmem) {
 }
 
 // TMA producer (one thread): Q rows of head h once, then key tiles of head h claimed one
-// at a time from the head's counter (shared by the head's CTAs) until none are left; the
-// stage after the last one carries tile id -1 and no data.
+// at a time from the head's counter (shared by the head's CTAs; the next claim is made while
+// the current tile's stage is awaited) until none are left; the stage after the last one
+// carries tile id -1 and no data.
 __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMap* tm_k,
                         const TcParams& p, int h, uint32_t* counter, bool load_q,
                         uint32_t* status) {
@@ -331,11 +369,13 @@ __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMa
   }
   int issued[kMaxStages];
   for (int i = 0; i < kMaxStages; ++i) issued[i] = 0;
+  uint32_t next = atomicAdd(counter, 1u);       // the next claim overlaps the stage wait
   for (int n = 0;; ++n) {
     const int st = n % p.nstages;
     const int use = n / p.nstages;
+    const uint32_t tile = next;
+    if (tile < uint32_t(p.T)) next = atomicAdd(counter, 1u);
     if (!bwait(bar_kempty(s, st), (use & 1) ^ 1, ab, p.wait_ns, status)) break;
-    const uint32_t tile = atomicAdd(counter, 1u);
     if (tile >= uint32_t(p.T)) {
       s.stile[st] = -1;
       mbar_arrive(bar_kfull(s, st));            // releases the id; no copy in flight
@@ -359,18 +399,25 @@ __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMa
   }
 }
 
-// MMA thread, start of its work: the optional stall hook (a wait on a barrier nothing
+// MMA warp (all lanes): bwait with one outcome for the whole warp.
+__device__ __forceinline__ bool wwait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                      uint64_t limit_ns, uint32_t* status) {
+  return __all_sync(0xffffffffu, bwait(bar, parity, abort_flag, limit_ns, status));
+}
+
+// MMA warp, start of its work: the optional stall hook (a wait on a barrier nothing
 // arrives on, to exercise the timeout path), then the wait for the Q rows.
 __device__ bool mma_start(const Smem& s, const TcParams& p, uint32_t* status) {
   volatile int* ab = s.abort_flag;
-  if ((p.flags & kFlagStallMma) && !bwait(bar_never(s), 0, ab, p.wait_ns, status)) return false;
-  return bwait(bar_qfull(s), 0, ab, p.wait_ns, status);
+  if ((p.flags & kFlagStallMma) && !wwait(bar_never(s), 0, ab, p.wait_ns, status)) return false;
+  return wwait(bar_qfull(s), 0, ab, p.wait_ns, status);
 }
 
 // Publishes the key tile of a TMEM slot use to the epilogue (the plain arrive on tfull
 // releases the store; the MMA commit is the barrier's second arrival).  Tile -1 ends the
 // epilogue's loop: both arrivals are made here.
-__device__ __forceinline__ void publish_slot(const Smem& s, int slot, int tile) {
+__device__ __forceinline__ void publish_slot(const Smem& s, int slot, int tile, uint32_t leader) {
+  if (!leader) return;
   s.utile[slot] = tile;
   if (tile < 0) mbar_arrive2(bar_tfull(s, slot));
   else mbar_arrive(bar_tfull(s, slot));
@@ -386,12 +433,13 @@ __device__ __forceinline__ void finish_claims(uint32_t* counter, uint32_t* finis
   }
 }
 
-// MMA thread, after an abort: a commit arrives on `drain` once every MMA this thread issued
-// has completed, so TMEM is not released under a running MMA.
-__device__ void mma_drain(const Smem& s, uint32_t* status) {
-  umma_commit(bar_drain(s));
+// MMA warp, after an abort: a commit arrives on `drain` once every MMA the warp issued has
+// completed, so TMEM is not released under a running MMA.
+__device__ void mma_drain(const Smem& s, uint32_t leader, uint32_t* status) {
+  umma_commit(bar_drain(s), leader);
   volatile int no_abort = 0;
   bwait(bar_drain(s), 0, &no_abort, kDrainNs, status);
+  __syncwarp();
 }
 
 // ---------------------------------------------------------------------------------------
@@ -459,39 +507,36 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   if (warp == 0) {
     if (lane == 0) produce(s, &tm_q, &tm_k, p, h, counter, true, ws.status);
   } else if (warp == 1) {
-    if (lane == 0) {
-      const uint32_t idesc = idesc_bf16(128, kTileKeys);
-      bool ok = mma_start(s, p, ws.status);
-      const uint32_t q0 = smem_u32(s.q), qhalf = uint32_t(s.qrows * 128);
-      for (int n = 0; ok; ++n) {
-        const int st = n % p.nstages;
-        if (!(ok = bwait(bar_kfull(s, st), (n / p.nstages) & 1, ab, p.wait_ns, ws.status))) break;
+    const uint32_t leader = elect_one();
+    const uint32_t idesc = idesc_bf16(128, kTileKeys);
+    bool ok = mma_start(s, p, ws.status);
+    const uint32_t q_lo = desc_lo(smem_u32(s.q)), qhalf = uint32_t(s.qrows * 128);
+    for (int n = 0; ok; ++n) {
+      const int st = n % p.nstages;
+      if (!(ok = wwait(bar_kfull(s, st), (n / p.nstages) & 1, ab, p.wait_ns, ws.status))) break;
+      tc_fence_after();
+      const int tile = s.stile[st];
+      const uint32_t k_lo = desc_lo(smem_u32(s.k + st * kStageBytes));
+#pragma unroll
+      for (int g = 0; g < NG; ++g) {
+        const int u = n * NG + g, slot = u & 1;
+        if (!(ok = wwait(bar_tempty(s, slot), ((u >> 1) & 1) ^ 1, ab, p.wait_ns, ws.status)))
+          break;
         tc_fence_after();
-        const int tile = s.stile[st];
-        const uint32_t k0 = smem_u32(s.k + st * kStageBytes);
-        for (int g = 0; g < NG; ++g) {
-          const int u = n * NG + g, slot = u & 1;
-          if (!(ok = bwait(bar_tempty(s, slot), ((u >> 1) & 1) ^ 1, ab, p.wait_ns, ws.status)))
-            break;
-          tc_fence_after();
-          publish_slot(s, slot, tile);
-          if (tile < 0) break;
-          for (int i = 0; i < 2 && 2 * g + i < NRT; ++i) {
-            const int rt = 2 * g + i;
-            for (int k = 0; k < 8; ++k) {
-              const uint32_t koff = uint32_t((k & 3) * 32), half = uint32_t(k >> 2);
-              const uint64_t a = sw128_desc(q0 + half * qhalf + uint32_t(rt) * kHalfBytes + koff);
-              const uint64_t bd = sw128_desc(k0 + half * kHalfBytes + koff);
-              umma_bf16(tmem + uint32_t(slot * 256 + i * kTileKeys), a, bd, idesc, k > 0 ? 1u : 0u);
-            }
-          }
-          umma_commit(bar_tfull(s, slot));
-        }
+        publish_slot(s, slot, tile, leader);
         if (tile < 0) break;
-        if (ok) umma_commit(bar_kempty(s, st));
+#pragma unroll
+        for (int i = 0; i < 2; ++i)
+          if (2 * g + i < NRT)
+            umma_k128(tmem + uint32_t(slot * 256 + i * kTileKeys),
+                      q_lo + uint32_t(2 * g + i) * (kHalfBytes >> 4), qhalf >> 4, k_lo,
+                      kHalfBytes >> 4, idesc, leader);
+        umma_commit(bar_tfull(s, slot), leader);
       }
-      if (!ok) mma_drain(s, ws.status);
+      if (tile < 0) break;
+      if (ok) umma_commit(bar_kempty(s, st), leader);
     }
+    if (!ok) mma_drain(s, leader, ws.status);
   } else {
     // Epilogue: the 4 warps of a TMEM lane quarter q share its 32 rows of every row tile
     // and split each slot's 128 keys into 4 blocks of 32.
@@ -590,36 +635,31 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   if (warp == 0) {
     if (lane == 0) produce(s, &tm_q, &tm_k, p, h, counter, true, ws.status);
   } else if (warp == 1) {
-    if (lane == 0) {
-      const uint32_t idesc = idesc_bf16(128, nn);
-      bool ok = mma_start(s, p, ws.status);
-      const uint32_t q0 = smem_u32(s.q), qhalf = uint32_t(s.qrows * 128);
-      for (int n = 0; ok; ++n) {
-        const int st = n % p.nstages;
-        if (!(ok = bwait(bar_kfull(s, st), (n / p.nstages) & 1, ab, p.wait_ns, ws.status))) break;
+    const uint32_t leader = elect_one();
+    const uint32_t idesc = idesc_bf16(128, nn);
+    bool ok = mma_start(s, p, ws.status);
+    const uint32_t q_lo = desc_lo(smem_u32(s.q)), qhalf = uint32_t(s.qrows * 128);
+    for (int n = 0; ok; ++n) {
+      const int st = n % p.nstages;
+      if (!(ok = wwait(bar_kfull(s, st), (n / p.nstages) & 1, ab, p.wait_ns, ws.status))) break;
+      tc_fence_after();
+      const int tile = s.stile[st];
+      const uint32_t k_lo = desc_lo(smem_u32(s.k + st * kStageBytes));
+      for (int c = 0; c < nch; ++c) {
+        const int u = n * nch + c, slot = u & 1;
+        if (!(ok = wwait(bar_tempty(s, slot), ((u >> 1) & 1) ^ 1, ab, p.wait_ns, ws.status)))
+          break;
         tc_fence_after();
-        const int tile = s.stile[st];
-        const uint32_t k0 = smem_u32(s.k + st * kStageBytes);
-        for (int c = 0; c < nch; ++c) {
-          const int u = n * nch + c, slot = u & 1;
-          if (!(ok = bwait(bar_tempty(s, slot), ((u >> 1) & 1) ^ 1, ab, p.wait_ns, ws.status)))
-            break;
-          tc_fence_after();
-          publish_slot(s, slot, tile);
-          if (tile < 0) break;
-          for (int k = 0; k < 8; ++k) {
-            const uint32_t koff = uint32_t((k & 3) * 32), half = uint32_t(k >> 2);
-            const uint64_t a = sw128_desc(k0 + half * kHalfBytes + koff);
-            const uint64_t b = sw128_desc(q0 + half * qhalf + uint32_t(c * nn) * 128 + koff);
-            umma_bf16(tmem + uint32_t(slot * 256), a, b, idesc, k > 0 ? 1u : 0u);
-          }
-          umma_commit(bar_tfull(s, slot));
-        }
+        publish_slot(s, slot, tile, leader);
         if (tile < 0) break;
-        if (ok) umma_commit(bar_kempty(s, st));
+        umma_k128(tmem + uint32_t(slot * 256), k_lo, kHalfBytes >> 4,
+                  q_lo + uint32_t(c * nn) * (128 >> 4), qhalf >> 4, idesc, leader);
+        umma_commit(bar_tfull(s, slot), leader);
       }
-      if (!ok) mma_drain(s, ws.status);
+      if (tile < 0) break;
+      if (ok) umma_commit(bar_kempty(s, st), leader);
     }
+    if (!ok) mma_drain(s, leader, ws.status);
   } else {
     const int ew = warp - 2, q = warp & 3, wi = ew >> 2;
     // Merge pass-1 partials of every window row into lse2 (log2 units): one online pass,
@@ -703,20 +743,40 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     finish_claims(counter, ws.sched + 3 * SGDKV_MAX_KV_HEADS + h, p.cph);
 }
 
-// scores = max-pool over [j - radius, j + radius] (clipped) of the four partial sums.
-__global__ void maxpool_sum_kernel(const float* __restrict__ raw, float* __restrict__ out,
-                                   int64_t L, int64_t n, int radius) {
-  const int64_t t = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (t >= n) return;
-  const int64_t j = t % L;
-  const float* r0 = raw + (t - j);
-  auto at = [&](int64_t i) { return (r0[i] + r0[n + i]) + (r0[2 * n + i] + r0[3 * n + i]); };
-  float m = at(j);
-  for (int s = 1; s <= radius; ++s) {
-    if (j - s >= 0) m = fmaxf(m, at(j - s));
-    if (j + s < L) m = fmaxf(m, at(j + s));
+// scores = max-pool over [j - radius, j + radius] (clipped to the row) of the sum of the
+// four partial-sum planes (Section 3.3's pooling of the window scores).  One block per
+// kPoolTile positions of one head: the plane sums of the tile and its halo are formed once
+// in shared memory with coalesced loads, then every output takes its window maximum there.
+constexpr int kPoolTile = 1024;
+constexpr int kPoolThreads = 256;
+constexpr int kMaxRadius = 31;                    // pool <= 63
+
+__global__ void __launch_bounds__(kPoolThreads)
+maxpool_sum_kernel(const float* __restrict__ raw, float* __restrict__ out, int64_t L,
+                   int64_t plane, int radius) {
+  __shared__ float sum[kPoolTile + 2 * kMaxRadius];
+  const int64_t tiles = ceil_div(L, kPoolTile);
+  const int h = int(blockIdx.x / tiles);
+  const int64_t base = (blockIdx.x % tiles) * kPoolTile;
+  const float* r0 = raw + int64_t(h) * L;
+  const int span = kPoolTile + 2 * radius;
+  for (int i = threadIdx.x; i < span; i += kPoolThreads) {
+    const int64_t j = base - radius + i;
+    float v = -INFINITY;
+    if (j >= 0 && j < L)
+      v = (__ldcg(r0 + j) + __ldcg(r0 + plane + j)) +
+          (__ldcg(r0 + 2 * plane + j) + __ldcg(r0 + 3 * plane + j));
+    sum[i] = v;
   }
-  out[t] = m;
+  __syncthreads();
+  float* o = out + int64_t(h) * L;
+  for (int i = threadIdx.x; i < kPoolTile; i += kPoolThreads) {
+    const int64_t j = base + i;
+    if (j >= L) break;
+    float m = sum[i + radius];
+    for (int k = 0; k < 2 * radius + 1; ++k) m = fmaxf(m, sum[i + k]);
+    o[j] = m;
+  }
 }
 
 // ---------------------------------------------------------------------------------------
@@ -763,6 +823,7 @@ uint32_t g_score_flags = 0;
 cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
                          int64_t L, int W, int pool, float* scores_out, const Ws& ws,
                          cudaStream_t stream) {
+  if (pool < 1 || pool / 2 > kMaxRadius) return cudaErrorInvalidValue;
   TcParams p{};
   p.Hkv = Hkv;
   p.G = Hq / Hkv;
@@ -817,11 +878,11 @@ cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq,
     KernelTimer t(SGDKV_KERNEL_SCORE_PASS2, stream);
     score_pass2_tc<<<grid, kThreads, smem2, stream>>>(tm_q, tm_k, p2, ws);
   }
-  const int64_t n = int64_t(Hkv) * L;
   {
     KernelTimer t(SGDKV_KERNEL_POOL, stream);
-    maxpool_sum_kernel<<<unsigned(ceil_div(n, 256)), 256, 0, stream>>>(ws.raw, scores_out, L, n,
-                                                                      pool / 2);
+    const unsigned blocks = unsigned(int64_t(Hkv) * ceil_div(L, kPoolTile));
+    maxpool_sum_kernel<<<blocks, kPoolThreads, 0, stream>>>(ws.raw, scores_out, L,
+                                                            int64_t(Hkv) * L, pool / 2);
   }
   note_launches(3);
   return cudaGetLastError();

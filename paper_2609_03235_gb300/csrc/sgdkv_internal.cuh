@@ -28,8 +28,8 @@ struct HeadTable {
 // Device views into the caller's workspace.
 struct Ws {
   uint32_t* status;      // sticky first device-side error (sgdkv_status)
-  uint32_t* sched;       // [4][SGDKV_MAX_KV_HEADS] key-tile counters and finish counts of
-                         // the two scoring passes (zero between launches)
+  uint32_t* sched;       // key-tile counters and finish counts of the two scoring passes
+                         // (kSched* offsets; zero between launches)
   float2* partial;       // [Hkv][kMaxScoreParts][kMaxRows] per-CTA (max, sum), log2 units
   float* raw;            // [4][Hkv][L] window scores before pooling, as four partial sums
   float* pooled;         // [Hkv][L] pooled scores (compress_layer scratch)
@@ -39,6 +39,11 @@ struct WsLayout {
   size_t status, partial, raw, pooled, total;   // status region: status word, then sched
 };
 constexpr size_t kSchedOffset = 1024;           // byte offset of Ws::sched in the status region
+// Ws::sched words: per head, the key-tile counters and finish counts of the two passes.
+constexpr int kSchedPass1Tiles = 0;
+constexpr int kSchedPass1Done = SGDKV_MAX_KV_HEADS;
+constexpr int kSchedPass2Tiles = 2 * SGDKV_MAX_KV_HEADS;
+constexpr int kSchedPass2Done = 3 * SGDKV_MAX_KV_HEADS;
 constexpr size_t kStatusRegionBytes = kSchedOffset + 4 * SGDKV_MAX_KV_HEADS * sizeof(uint32_t);
 
 __host__ __device__ inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }

@@ -48,7 +48,7 @@ SCORE_SHAPES = [
 
 
 @pytest.mark.parametrize("Hq,Hkv,L,W", SCORE_SHAPES)
-@pytest.mark.parametrize("pool", [1, 7])
+@pytest.mark.parametrize("pool", [1, 7, 63])
 def test_score_parity(dev, Hq, Hkv, L, W, pool):
     wl = synth.tiny_workload(Hq=Hq, Hkv=Hkv, d=128, L=L, W=W, n_salient=min(8, max(0, L - W - 4)))
     inp = synth.tiny_inputs(wl, tag=200 + L)
