@@ -16,12 +16,14 @@
 //     rows (four warps per key), written to four partial-sum planes of the raw buffer.
 //   pool (maxpool_sum_kernel): scores = max-pool of the sum of the four planes.
 //
-// CTA roles (576 threads): warp 0 lane 0 issues TMA loads (Q_h once, K tiles of 128 keys
-// through a ring of shared-memory stages); warp 1 allocates the 512 TMEM columns
-// and its lane 0 issues the MMAs; warps 2..17 are the epilogue (four per TMEM lane
-// quarter).  An epilogue warp loads all its TMEM columns of a slot, releases the slot,
-// then does the arithmetic, so the MMAs of the next slot overlap it.  Each CTA owns one KV
-// head and a contiguous range of key tiles.  Every wait on an mbarrier is bounded in time:
+// CTA roles (640 threads): warp 2 lane 0 issues TMA loads (Q_h once, K tiles of 128 keys
+// through a ring of shared-memory stages); warp 3 allocates the 512 TMEM columns and its
+// elected lane issues the MMAs; warps 4..19 are the epilogue (four per TMEM lane quarter);
+// warps 0 and 1 idle, so that the control warps share sub-partitions with the lane
+// quarters that carry less epilogue work.  An epilogue warp loads all its TMEM columns of a
+// slot, releases the slot, then does the arithmetic, so the MMAs of the next slot overlap
+// it.  Each CTA owns one KV head and claims its key tiles from a counter shared by the
+// head's CTAs.  Every wait on an mbarrier is bounded in time:
 // on expiry the kernel records SGDKV_ERR_TIMEOUT, all roles leave their loops, in-flight
 // copies and MMAs are drained (again bounded) and TMEM is freed.
 #include <cuda.h>
@@ -32,9 +34,16 @@
 namespace sgdkv {
 namespace {
 
-constexpr int kThreads = 576;                     // 18 warps
+// Warp roles.  Warp w runs on SM sub-partition w % 4 and reaches TMEM lanes 32 * (w % 4)..
+// The producer and the MMA warp sit on sub-partitions 2 and 3: with G*W rows padded to
+// 128-row tiles, the extra (partial) row tile of pass 1 lands on lane quarters 0 and 1, so
+// the four sub-partitions carry about the same load.  Warps 0 and 1 have no role.
+constexpr int kProducerWarp = 2;
+constexpr int kMmaWarp = 3;
+constexpr int kFirstEpiWarp = 4;                  // warps 4..19: epilogue, four per quarter
+constexpr int kThreads = 640;                     // 20 warps
 constexpr int kEpiWarps = 16;
-constexpr int kMaxRegs = 96;   // 18 warps: 5 warps x 96 x 32 fit one 16K-register SM sub-partition
+constexpr int kMaxRegs = 96;   // 5 warps x 96 x 32 fit one 16K-register SM sub-partition
 constexpr int kTileKeys = 128;
 constexpr uint32_t kTmemCols = 512;
 constexpr int kStageBytes = kTileKeys * 256;      // 32 KB: two 128-byte column halves
@@ -327,7 +336,7 @@ __device__ __forceinline__ uint32_t setup(const Smem& s, int nstages, uint32_t q
     *s.abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 1) {
+  if (warp == kMmaWarp) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_u32(s.tmem_slot)),
                  "r"(kTmemCols)
@@ -344,7 +353,7 @@ __device__ __forceinline__ void teardown(uint32_t tmem) {
   __syncwarp();
   tc_fence_before();
   __syncthreads();
-  if ((threadIdx.x >> 5) == 1) {
+  if ((threadIdx.x >> 5) == kMmaWarp) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                  "r"(kTmemCols)
@@ -504,9 +513,9 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   const uint32_t tmem = setup(s, p.nstages, 1);
   volatile int* ab = s.abort_flag;
 
-  if (warp == 0) {
+  if (warp == kProducerWarp) {
     if (lane == 0) produce(s, &tm_q, &tm_k, p, h, counter, true, ws.status);
-  } else if (warp == 1) {
+  } else if (warp == kMmaWarp) {
     const uint32_t leader = elect_one();
     const uint32_t idesc = idesc_bf16(128, kTileKeys);
     bool ok = mma_start(s, p, ws.status);
@@ -537,10 +546,10 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
       if (ok) umma_commit(bar_kempty(s, st), leader);
     }
     if (!ok) mma_drain(s, leader, ws.status);
-  } else {
+  } else if (warp >= kFirstEpiWarp) {
     // Epilogue: the 4 warps of a TMEM lane quarter q share its 32 rows of every row tile
     // and split each slot's 128 keys into 4 blocks of 32.
-    const int q = warp & 3, wi = (warp - 2) >> 2;
+    const int q = warp & 3, wi = (warp - kFirstEpiWarp) >> 2;
     const int lim_base = int(p.L - p.W);       // Hkv * L < 2^31
     float m[NRT], Z[NRT];
     int lim[NRT];
@@ -632,9 +641,9 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   const int nch = p.GW > 256 ? 2 : 1;            // N chunks of the window rows per tile
   const int nn = p.GW / nch;                     // MMA N
 
-  if (warp == 0) {
+  if (warp == kProducerWarp) {
     if (lane == 0) produce(s, &tm_q, &tm_k, p, h, counter, true, ws.status);
-  } else if (warp == 1) {
+  } else if (warp == kMmaWarp) {
     const uint32_t leader = elect_one();
     const uint32_t idesc = idesc_bf16(128, nn);
     bool ok = mma_start(s, p, ws.status);
@@ -660,21 +669,22 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
       if (ok) umma_commit(bar_kempty(s, st), leader);
     }
     if (!ok) mma_drain(s, leader, ws.status);
-  } else {
-    const int ew = warp - 2, q = warp & 3, wi = ew >> 2;
+  } else if (warp >= kFirstEpiWarp) {
+    const int ew = warp - kFirstEpiWarp, q = warp & 3, wi = ew >> 2;
     // Merge pass-1 partials of every window row into lse2 (log2 units): one online pass,
-    // sixteen independent loads in flight per step.
+    // twenty independent loads in flight per step.
     for (int r = ew * 32 + lane; r < p.GW; r += kEpiWarps * 32) {
       const float2* pp = ws.partial + int64_t(h) * kMaxScoreParts * kMaxRows + r;
       float M = -INFINITY, S = 0.f;
-      for (int i0 = 0; i0 < p.nparts; i0 += 16) {
-        float2 v[16];
+      constexpr int kB = 20;
+      for (int i0 = 0; i0 < p.nparts; i0 += kB) {
+        float2 v[kB];
 #pragma unroll
-        for (int i = 0; i < 16; ++i)
+        for (int i = 0; i < kB; ++i)
           v[i] = i0 + i < p.nparts ? __ldcg(pp + int64_t(i0 + i) * kMaxRows)
                                    : make_float2(-INFINITY, 0.f);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
+        for (int i = 0; i < kB; ++i) {
           if (v[i].x == -INFINITY) continue;
           const float mn = fmaxf(M, v[i].x);
           S = (M == -INFINITY ? 0.f : S * ex2(M - mn)) + v[i].y * ex2(v[i].x - mn);
