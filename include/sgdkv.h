@@ -120,6 +120,24 @@ SGDKV_API sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq,
                          void* workspace, size_t ws_bytes, void* stream);
 
 /*
+ * sgdkv_score with scoring flags.  flags == 0 is sgdkv_score.
+ *
+ * SGDKV_SCORE_PROXY_QUERY: the W rows of q_win per query head are an external query (the
+ * proxy-query setting of the paper's query ablation, Section "Ablation Study: Impact of
+ * Query on Token Selection", Table 3: a fixed task-agnostic prompt stands in for the
+ * unknown question).  Such queries come after the whole context, so every row sees all L
+ * keys: no causal mask, raw[h][j] = sum_{g,w} softmax_j over all L keys.  (The
+ * query-unaware setting of the same ablation is ordinary scoring of a context that ends
+ * before the question: flags == 0 with that L.)
+ * Unknown flag bits: INVALID_ARG.  Other arguments and errors as sgdkv_score.
+ */
+#define SGDKV_SCORE_PROXY_QUERY 1u
+SGDKV_API sgdkv_status sgdkv_score_ex(const void* q_win, const void* K, int32_t Hq, int32_t Hkv,
+                                      int64_t L, int32_t d, int32_t W, int32_t pool,
+                                      uint32_t flags, float* scores_out, void* workspace,
+                                      size_t ws_bytes, void* stream);
+
+/*
  * sgdkv_score without a workspace argument, for callers that cannot allocate device
  * memory (for example code running where the allocator is owned by someone else, or a
  * plugin that may only receive tensors).  No counterpart in the paper: the computation

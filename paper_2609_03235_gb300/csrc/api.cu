@@ -170,19 +170,27 @@ size_t sgdkv_workspace_bytes(int32_t Hq, int32_t Hkv, int64_t L, int32_t d, int3
   return workspace_layout(Hkv, L).total;
 }
 
-sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq, int32_t Hkv, int64_t L,
-                         int32_t d, int32_t W, int32_t pool, float* scores_out,
-                         void* workspace, size_t ws_bytes, void* stream) {
+sgdkv_status sgdkv_score_ex(const void* q_win, const void* K, int32_t Hq, int32_t Hkv, int64_t L,
+                            int32_t d, int32_t W, int32_t pool, uint32_t flags, float* scores_out,
+                            void* workspace, size_t ws_bytes, void* stream) {
   if (!q_win || !K || !scores_out) return SGDKV_ERR_INVALID_ARG;
   if (!aligned16(q_win) || !aligned16(K) || !aligned16(scores_out)) return SGDKV_ERR_INVALID_ARG;
+  if (flags & ~SGDKV_SCORE_PROXY_QUERY) return SGDKV_ERR_INVALID_ARG;
   sgdkv_status s = check_score_shape(Hq, Hkv, L, d, W);
   if (s != SGDKV_OK) return s;
   if ((s = check_pool(pool)) != SGDKV_OK) return s;
   if ((s = check_workspace(workspace, ws_bytes, Hkv, L)) != SGDKV_OK) return s;
   const Ws ws = workspace_view(workspace, workspace_layout(Hkv, L));
   return from_cuda(launch_score(static_cast<const __nv_bfloat16*>(q_win),
-                                static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, pool,
+                                static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, pool, flags,
                                 scores_out, ws, static_cast<cudaStream_t>(stream)));
+}
+
+sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq, int32_t Hkv, int64_t L,
+                         int32_t d, int32_t W, int32_t pool, float* scores_out,
+                         void* workspace, size_t ws_bytes, void* stream) {
+  return sgdkv_score_ex(q_win, K, Hq, Hkv, L, d, W, pool, 0u, scores_out, workspace, ws_bytes,
+                        stream);
 }
 
 sgdkv_status sgdkv_score_static(const void* q_win, const void* K, int32_t Hq, int32_t Hkv,
@@ -205,7 +213,7 @@ sgdkv_status sgdkv_score_static(const void* q_win, const void* K, int32_t Hq, in
   cudaError_t e = cudaMemsetAsync(ws.status, 0, kStatusRegionBytes, st);
   if (e != cudaSuccess) return from_cuda(e);
   e = launch_score(static_cast<const __nv_bfloat16*>(q_win), static_cast<const __nv_bfloat16*>(K),
-                   Hq, Hkv, L, W, pool, scores_out, ws, st);
+                   Hq, Hkv, L, W, pool, 0u, scores_out, ws, st);
   if (e != cudaSuccess) return from_cuda(e);
   if (status_out) {
     e = cudaMemcpyAsync(status_out, ws.status, sizeof(uint32_t), cudaMemcpyDeviceToDevice, st);
@@ -261,7 +269,7 @@ sgdkv_status sgdkv_compress_layer(const void* q_win, const void* K, const void* 
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   float* pooled = scores_out ? scores_out : ws.pooled;
   cudaError_t e = launch_score(static_cast<const __nv_bfloat16*>(q_win),
-                               static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, pool,
+                               static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, pool, 0u,
                                pooled, ws, st);
   if (e != cudaSuccess) return from_cuda(e);
   return from_cuda(launch_compact(static_cast<const __nv_bfloat16*>(K),

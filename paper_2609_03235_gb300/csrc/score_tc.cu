@@ -66,6 +66,7 @@ struct TcParams {
   int nstages;    // K ring depth
   int nparts;     // pass 2: partial slots per head written by pass 1
   float scale2;   // log2(e) / sqrt(d)
+  int causal;     // 1: window row w sees keys <= L - W + w; 0: every row sees all L keys
   uint64_t wait_ns;
   uint32_t flags;
 };
@@ -550,7 +551,8 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     // Epilogue: the 4 warps of a TMEM lane quarter q share its 32 rows of every row tile
     // and split each slot's 128 keys into 4 blocks of 32.
     const int q = warp & 3, wi = (warp - kFirstEpiWarp) >> 2;
-    const int lim_base = int(p.L - p.W);       // Hkv * L < 2^31
+    // keys above a row's limit are masked; lim_base: the lowest limit of any row
+    const int lim_base = p.causal ? int(p.L - p.W) : int(p.L - 1);   // Hkv * L < 2^31
     float m[NRT], Z[NRT];
     int lim[NRT];
     bool valid[NRT];
@@ -559,7 +561,7 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
       m[rt] = -INFINITY;
       Z[rt] = 0.f;
       valid[rt] = rt * 128 + 32 * q < p.GW;                  // warp-uniform
-      lim[rt] = lim_base + (rt * 128 + 32 * q + lane) % p.W;
+      lim[rt] = p.causal ? lim_base + (rt * 128 + 32 * q + lane) % p.W : lim_base;
     }
     bool ok = true;
     for (int n = 0; ok; ++n) {
@@ -699,7 +701,7 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     // are dealt to them in blocks of 16 columns, round robin over the whole tile.
     const int gpc = nn / 16;                     // 16-column blocks per chunk (<= 16)
     float* raw_out = ws.raw + int64_t(wi) * p.Hkv * p.L + int64_t(h) * p.L;
-    const int lim_base = int(p.L - p.W);
+    const int lim_base = p.causal ? int(p.L - p.W) : int(p.L - 1);   // lowest row limit
     bool ok = true;
     for (int n = 0; ok; ++n) {
       int j = 0;
@@ -734,7 +736,7 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
           if (masked) {                            // rows that cannot see key j drop out
 #pragma unroll
             for (int e = 0; e < 16; ++e)
-              if (j > lim_base + (r0 + e) % p.W) v[k][e] = 0xff800000u;
+              if (j > (p.causal ? lim_base + (r0 + e) % p.W : lim_base)) v[k][e] = 0xff800000u;
           }
           const float4* nl = reinterpret_cast<const float4*>(lse2 + r0);
 #pragma unroll
@@ -831,8 +833,8 @@ uint64_t g_score_wait_ns = 2000000000ull;
 uint32_t g_score_flags = 0;
 
 cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
-                         int64_t L, int W, int pool, float* scores_out, const Ws& ws,
-                         cudaStream_t stream) {
+                         int64_t L, int W, int pool, uint32_t flags, float* scores_out,
+                         const Ws& ws, cudaStream_t stream) {
   if (pool < 1 || pool / 2 > kMaxRadius) return cudaErrorInvalidValue;
   TcParams p{};
   p.Hkv = Hkv;
@@ -849,6 +851,7 @@ cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq,
   p.nparts = p.cph;
   if (p.nparts > kMaxScoreParts) return cudaErrorInvalidConfiguration;
   p.scale2 = kLog2e / sqrtf(float(kD));
+  p.causal = (flags & SGDKV_SCORE_PROXY_QUERY) ? 0 : 1;
   p.wait_ns = g_score_wait_ns;
   p.flags = g_score_flags;
 

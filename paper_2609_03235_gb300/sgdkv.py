@@ -21,7 +21,7 @@ EXPORTED = ("sgdkv_status_string", "sgdkv_version", "sgdkv_allocate_budgets",
             "sgdkv_workspace_bytes", "sgdkv_score", "sgdkv_compact", "sgdkv_compress_layer",
             "sgdkv_last_error", "sgdkv_launch_count", "sgdkv_debug_set_score_hooks",
             "sgdkv_last_cuda_error_string", "sgdkv_score_static",
-            "sgdkv_debug_enable_kernel_timing", "sgdkv_debug_kernel_timing")
+            "sgdkv_debug_enable_kernel_timing", "sgdkv_debug_kernel_timing", "sgdkv_score_ex")
 
 
 class LibraryMissing(RuntimeError):
@@ -68,6 +68,9 @@ def lib():
         L.sgdkv_last_error.argtypes = [_P, _P]
         L.sgdkv_launch_count.restype = ctypes.c_uint64
         L.sgdkv_last_cuda_error_string.restype = ctypes.c_char_p
+        L.sgdkv_score_ex.restype = ctypes.c_int
+        L.sgdkv_score_ex.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, _I32, ctypes.c_uint32,
+                                     _P, _P, _SZ, _P]
         L.sgdkv_score_static.restype = ctypes.c_int
         L.sgdkv_score_static.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, _I32, _P, _P, _P]
         L.sgdkv_debug_set_score_hooks.restype = None
@@ -129,12 +132,23 @@ def make_workspace(Hq: int, Hkv: int, L: int, W: int, device="cuda", d: int = 12
     return torch.zeros(n, dtype=torch.uint8, device=device)
 
 
-def sgdkv_score(q_win, K, W: int, pool: int, scores_out, workspace, stream=None):
+SCORE_PROXY_QUERY = 1
+
+
+def sgdkv_score(q_win, K, W: int, pool: int, scores_out, workspace, stream=None, flags: int = 0):
+    """Window scores (flags 0: causal observation window) or, with SCORE_PROXY_QUERY,
+    scores of external queries that see every key (sgdkv_score_ex)."""
     Hq, W_, d = q_win.shape
     Hkv, L, _ = K.shape
-    st = lib().sgdkv_score(_ptr(q_win), _ptr(K), Hq, Hkv, L, d, W, pool, _ptr(scores_out),
-                           _ptr(workspace), workspace.numel(), _stream(stream))
-    _check(st, "sgdkv_score")
+    if flags == 0:
+        st = lib().sgdkv_score(_ptr(q_win), _ptr(K), Hq, Hkv, L, d, W, pool, _ptr(scores_out),
+                               _ptr(workspace), workspace.numel(), _stream(stream))
+        _check(st, "sgdkv_score")
+        return
+    st = lib().sgdkv_score_ex(_ptr(q_win), _ptr(K), Hq, Hkv, L, d, W, pool, int(flags),
+                              _ptr(scores_out), _ptr(workspace), workspace.numel(),
+                              _stream(stream))
+    _check(st, "sgdkv_score_ex")
 
 
 def sgdkv_score_static(q_win, K, W: int, pool: int, scores_out, status_out=None, stream=None):

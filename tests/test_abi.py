@@ -119,6 +119,12 @@ def test_score_rejects_bad_args_before_device_work():
     assert L.sgdkv_score(p, p, 28, 4, 1024, 128, 32, 6, p, p, 1 << 30, None) == sg.ERR_INVALID_ARG
     # workspace too small
     assert L.sgdkv_score(p, p, 28, 4, 1024, 128, 32, 7, p, p, 16, None) == sg.ERR_WORKSPACE
+    # sgdkv_score_ex: unknown flag bits, then the same checks as sgdkv_score
+    assert L.sgdkv_score_ex(p, p, 28, 4, 1024, 128, 32, 7, 2, p, p, 1 << 30, None) == sg.ERR_INVALID_ARG
+    assert L.sgdkv_score_ex(p, p, 28, 4, 1024, 128, 32, 6, sg.SCORE_PROXY_QUERY, p, p, 1 << 30,
+                            None) == sg.ERR_INVALID_ARG
+    assert L.sgdkv_score_ex(p, p, 28, 4, 1024, 128, 32, 7, sg.SCORE_PROXY_QUERY, p, p, 16,
+                            None) == sg.ERR_WORKSPACE
 
 
 def test_compact_rejects_bad_budgets():

@@ -65,6 +65,38 @@ def test_score_parity(dev, Hq, Hkv, L, W, pool):
     assert ok.all(), f"{(~ok).sum()} of {ok.size} off; worst {np.max(np.abs(got - exp))}"
 
 
+PROXY_SHAPES = [
+    # Hq, Hkv, L, W    (W external query rows per query head; every row sees all L keys)
+    (14, 2, 1000, 32),
+    (28, 4, 3000, 64),
+    (16, 2, 2049, 64),
+    (1, 1, 300, 32),
+    (9, 1, 1000, 32),
+    (28, 4, 20000, 64),
+]
+
+
+@pytest.mark.parametrize("Hq,Hkv,L,W", PROXY_SHAPES)
+@pytest.mark.parametrize("pool", [1, 7])
+def test_proxy_query_score_parity(dev, Hq, Hkv, L, W, pool):
+    """Proxy-query scoring (no causal mask) against the oracle's non-causal scores."""
+    wl = synth.tiny_workload(Hq=Hq, Hkv=Hkv, d=128, L=L, W=W, n_salient=min(8, max(0, L - W - 4)))
+    inp = synth.tiny_inputs(wl, tag=600 + L)
+    q, K, _ = _upload(inp, dev)
+    ws = sg.make_workspace(Hq, Hkv, L, W, dev)
+    out = torch.empty((Hkv, L), dtype=torch.float32, device=dev)
+    sg.sgdkv_score(q, K, W, pool, out, ws, flags=sg.SCORE_PROXY_QUERY)
+    torch.cuda.synchronize()
+    assert sg.sgdkv_last_error(ws) == sg.OK
+    exp = O.max_pool(O.window_scores(inp["q"], inp["K"], causal=False), pool)
+    got = out.cpu().numpy()
+    ok = _within(got, exp)
+    assert ok.all(), f"{(~ok).sum()} of {ok.size} off; worst {np.max(np.abs(got - exp))}"
+    # every row sees every key: the raw scores of a head sum to G*W
+    if pool == 1:
+        assert np.allclose(got.astype(np.float64).sum(axis=1), Hq // Hkv * W, rtol=1e-4)
+
+
 def _tie_heavy_scores(rng, Hkv, L):
     return (rng.integers(0, 6, size=(Hkv, L)) * 0.125).astype(np.float32)
 

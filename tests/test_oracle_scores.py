@@ -21,13 +21,27 @@ def _f(x):
 
 
 @pytest.mark.parametrize("Hq,Hkv,L,W,d", [(4, 2, 50, 8, 16), (7, 1, 33, 32, 8), (8, 8, 9, 1, 4)])
-def test_rows_sum_to_one(Hq, Hkv, L, W, d):
+@pytest.mark.parametrize("causal", [True, False])
+def test_rows_sum_to_one(Hq, Hkv, L, W, d, causal):
     rng = np.random.default_rng(L)
     q = rng.standard_normal((Hq, W, d))
     k = rng.standard_normal((Hkv, L, d)) * 3
-    raw = O.window_scores(q, k).astype(np.float64)
+    raw = O.window_scores(q, k, causal=causal).astype(np.float64)
     G = Hq // Hkv
     assert np.allclose(raw.sum(axis=1), G * W, rtol=1e-6)
+
+
+def test_non_causal_sees_the_last_keys_from_every_row():
+    """Without the causal mask the first window row's softmax covers keys beyond L - W:
+    a key planted at the last position draws mass from every row (it would draw none from
+    rows w < W - 1 under the causal mask)."""
+    L, W, d = 40, 8, 16
+    q = np.zeros((1, W, d)); q[:, :, 0] = 1.0
+    k = np.zeros((1, L, d)); k[0, L - 1, 0] = 20.0 * np.sqrt(d)
+    nc = O.window_scores(q, k, causal=False).astype(np.float64)
+    c = O.window_scores(q, k, causal=True).astype(np.float64)
+    assert nc[0, L - 1] > W - 1e-3                   # every row puts ~all its mass on it
+    assert c[0, L - 1] < 1 + 1e-3                    # only the last row sees it
 
 
 @pytest.mark.parametrize("causal", [True, False])
