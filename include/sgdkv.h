@@ -120,22 +120,43 @@ SGDKV_API sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq,
                          void* workspace, size_t ws_bytes, void* stream);
 
 /*
- * sgdkv_score with scoring flags.  flags == 0 is sgdkv_score.
+ * sgdkv_score with scoring flags.  flags == 0 (and head_weights NULL) is sgdkv_score.
  *
  * SGDKV_SCORE_PROXY_QUERY: the W rows of q_win per query head are an external query (the
  * proxy-query setting of the paper's query ablation, Section "Ablation Study: Impact of
  * Query on Token Selection", Table 3: a fixed task-agnostic prompt stands in for the
  * unknown question).  Such queries come after the whole context, so every row sees all L
- * keys: no causal mask, raw[h][j] = sum_{g,w} softmax_j over all L keys.  (The
- * query-unaware setting of the same ablation is ordinary scoring of a context that ends
- * before the question: flags == 0 with that L.)
- * Unknown flag bits: INVALID_ARG.  Other arguments and errors as sgdkv_score.
+ * keys: no causal mask.  (The query-unaware setting of the same ablation is ordinary
+ * scoring of a context that ends before the question: flags without this bit, that L.)
+ *
+ * Aggregation over the GQA group (flag bits 1-2; the appendix's head configuration
+ * variants, "Ipt." rows of its ablation table).  With A_g[j] the cumulative window
+ * attention of query head g of the group (sum over its W rows of the softmax) and w_g its
+ * summarization score, head_weights[q] = w of query head q:
+ *   SGDKV_SCORE_AGG_SUM      (0)  raw[j] = sum_g A_g[j]            (sgdkv_score)
+ *   SGDKV_SCORE_AGG_IPT_MAX       raw[j] = max_g w_g A_g[j]        ("Ipt., Max")
+ *   SGDKV_SCORE_AGG_IPT_MEAN      raw[j] = mean_g w_g A_g[j]       ("Ipt., Mean")
+ *   SGDKV_SCORE_AGG_IPT_ONLY      raw[j] = A_g*[j], g* the group's highest w (lower g on
+ *                                 ties)                            ("Ipt., Only")
+ * then max-pooling as in sgdkv_score.  head_weights: device fp32 [Hq], finite and >= 0
+ * (required for the IPT modes, ignored otherwise); a negative or non-finite weight is
+ * found on the device, records SGDKV_ERR_INVALID_ARG in the workspace status word
+ * (sgdkv_last_error) and its head contributes nothing.  SGDKV_SCORE_AGG_IPT_MAX needs
+ * W in {16, 32, 48, 64} and G <= 8 (UNSUPPORTED otherwise).
+ * Unknown flag bits, or an IPT mode without head_weights: INVALID_ARG.  Other arguments and
+ * errors as sgdkv_score.
  */
 #define SGDKV_SCORE_PROXY_QUERY 1u
+#define SGDKV_SCORE_AGG_SUM (0u << 1)
+#define SGDKV_SCORE_AGG_IPT_MAX (1u << 1)
+#define SGDKV_SCORE_AGG_IPT_MEAN (2u << 1)
+#define SGDKV_SCORE_AGG_IPT_ONLY (3u << 1)
+#define SGDKV_SCORE_AGG_MASK (3u << 1)
 SGDKV_API sgdkv_status sgdkv_score_ex(const void* q_win, const void* K, int32_t Hq, int32_t Hkv,
                                       int64_t L, int32_t d, int32_t W, int32_t pool,
-                                      uint32_t flags, float* scores_out, void* workspace,
-                                      size_t ws_bytes, void* stream);
+                                      uint32_t flags, const float* head_weights,
+                                      float* scores_out, void* workspace, size_t ws_bytes,
+                                      void* stream);
 
 /*
  * sgdkv_score without a workspace argument, for callers that cannot allocate device

@@ -17,6 +17,11 @@ Steps and the passages they follow (SGD-KV, "Summarization Guided KV Cache Compr
   attention of a final observation window, SnapKV-style): softmax over the causal keys of
   each window query, summed over the window and over the query heads of the KV head's
   GQA group; scale 1/sqrt(d).
+* ``window_scores_ipt``: Appendix, "Head Configurations Variants" (last part of the
+  ablation table): per query head g, its cumulative window attention A_g[j] weighted by
+  the head's summarization score w_g, combined within the GQA group by max ("Ipt., Max")
+  or mean ("Ipt., Mean"), or the attention of the group's highest-scoring head alone
+  ("Ipt., Only"; ties: lower head).
 * ``max_pool``: 1-D max smoothing of the window scores, odd kernel, stride 1, same length,
   the window clipped at the sequence ends.  The paper is silent on pooling; the
   smoothing step is part of the stated problem of this library.
@@ -35,6 +40,7 @@ import math
 import numpy as np
 
 GREEDY, PROPORTIONAL, THRESHOLD = 0, 1, 2
+AGG_SUM, AGG_IPT_MAX, AGG_IPT_MEAN, AGG_IPT_ONLY = 0, 1, 2, 3
 
 
 # ----------------------------------------------------------------------------------------
@@ -195,6 +201,56 @@ def window_scores(q_win, K, causal: bool = True) -> np.ndarray:
             p = e / e.sum(axis=1, keepdims=True)
             raw[h] += p.sum(axis=0)
     return raw.astype(np.float32)
+
+
+def head_window_attention(q_win, K, causal: bool = True) -> np.ndarray:
+    """A[q, j] = sum_{w < W} softmax_j(q[q, w] . K[q // G, j] / sqrt(d)) for every query head
+    q (same softmax and mask as ``window_scores``); float64 [Hq, L]."""
+    q = bf16_bits_to_f64(q_win) if np.asarray(q_win).dtype == np.uint16 else np.asarray(q_win, np.float64)
+    k = bf16_bits_to_f64(K) if np.asarray(K).dtype == np.uint16 else np.asarray(K, np.float64)
+    Hq, W, d = q.shape
+    Hkv, L, _ = k.shape
+    G = Hq // Hkv
+    A = np.zeros((Hq, L), dtype=np.float64)
+    pos = np.arange(L)
+    for qh in range(Hq):
+        logits = (q[qh] @ k[qh // G].T) / math.sqrt(d)            # [W, L]
+        if causal:
+            visible = pos[None, :] <= (L - W + np.arange(W))[:, None]
+            logits = np.where(visible, logits, -np.inf)
+        m = logits.max(axis=1, keepdims=True)
+        e = np.exp(logits - m)
+        A[qh] = (e / e.sum(axis=1, keepdims=True)).sum(axis=0)
+    return A
+
+
+def window_scores_ipt(q_win, K, head_weights, mode: int, causal: bool = True) -> np.ndarray:
+    """Summarization-weighted GQA aggregation of the window attention (Appendix, head
+    configuration variants).  head_weights: [Hq] non-negative summarization scores of the
+    layer's query heads.  mode AGG_IPT_MAX: max_g w_g A_g; AGG_IPT_MEAN: mean_g w_g A_g;
+    AGG_IPT_ONLY: A_{g*} with g* the group's highest-scoring head (lower index on ties);
+    AGG_SUM: sum_g A_g (``window_scores``).  Returns float32 [Hkv, L]."""
+    A = head_window_attention(q_win, K, causal)
+    w = np.asarray(head_weights, dtype=np.float64)
+    Hq, L = A.shape
+    Hkv = np.asarray(K).shape[0]
+    G = Hq // Hkv
+    if w.shape != (Hq,) or not np.all(np.isfinite(w)) or np.any(w < 0):
+        raise ValueError("head_weights must be Hq finite non-negative values")
+    out = np.zeros((Hkv, L), dtype=np.float64)
+    for h in range(Hkv):
+        grp = slice(h * G, (h + 1) * G)
+        if mode == AGG_SUM:
+            out[h] = A[grp].sum(axis=0)
+        elif mode == AGG_IPT_MAX:
+            out[h] = (w[grp, None] * A[grp]).max(axis=0)
+        elif mode == AGG_IPT_MEAN:
+            out[h] = (w[grp, None] * A[grp]).mean(axis=0)
+        elif mode == AGG_IPT_ONLY:
+            out[h] = A[h * G + int(np.argmax(w[grp]))]
+        else:
+            raise ValueError("unknown aggregation mode")
+    return out.astype(np.float32)
 
 
 def max_pool(raw, kernel: int = 7) -> np.ndarray:

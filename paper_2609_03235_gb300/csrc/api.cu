@@ -171,26 +171,32 @@ size_t sgdkv_workspace_bytes(int32_t Hq, int32_t Hkv, int64_t L, int32_t d, int3
 }
 
 sgdkv_status sgdkv_score_ex(const void* q_win, const void* K, int32_t Hq, int32_t Hkv, int64_t L,
-                            int32_t d, int32_t W, int32_t pool, uint32_t flags, float* scores_out,
-                            void* workspace, size_t ws_bytes, void* stream) {
+                            int32_t d, int32_t W, int32_t pool, uint32_t flags,
+                            const float* head_weights, float* scores_out, void* workspace,
+                            size_t ws_bytes, void* stream) {
   if (!q_win || !K || !scores_out) return SGDKV_ERR_INVALID_ARG;
   if (!aligned16(q_win) || !aligned16(K) || !aligned16(scores_out)) return SGDKV_ERR_INVALID_ARG;
-  if (flags & ~SGDKV_SCORE_PROXY_QUERY) return SGDKV_ERR_INVALID_ARG;
+  if (flags & ~(SGDKV_SCORE_PROXY_QUERY | SGDKV_SCORE_AGG_MASK)) return SGDKV_ERR_INVALID_ARG;
+  const uint32_t agg = flags & SGDKV_SCORE_AGG_MASK;
+  if (agg != SGDKV_SCORE_AGG_SUM && !head_weights) return SGDKV_ERR_INVALID_ARG;
   sgdkv_status s = check_score_shape(Hq, Hkv, L, d, W);
   if (s != SGDKV_OK) return s;
+  if (agg == SGDKV_SCORE_AGG_IPT_MAX && (W % 16 != 0 || W > 64 || Hq / Hkv > 8))
+    return SGDKV_ERR_UNSUPPORTED;
   if ((s = check_pool(pool)) != SGDKV_OK) return s;
   if ((s = check_workspace(workspace, ws_bytes, Hkv, L)) != SGDKV_OK) return s;
   const Ws ws = workspace_view(workspace, workspace_layout(Hkv, L));
   return from_cuda(launch_score(static_cast<const __nv_bfloat16*>(q_win),
                                 static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, pool, flags,
-                                scores_out, ws, static_cast<cudaStream_t>(stream)));
+                                agg == SGDKV_SCORE_AGG_SUM ? nullptr : head_weights, scores_out,
+                                ws, static_cast<cudaStream_t>(stream)));
 }
 
 sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq, int32_t Hkv, int64_t L,
                          int32_t d, int32_t W, int32_t pool, float* scores_out,
                          void* workspace, size_t ws_bytes, void* stream) {
-  return sgdkv_score_ex(q_win, K, Hq, Hkv, L, d, W, pool, 0u, scores_out, workspace, ws_bytes,
-                        stream);
+  return sgdkv_score_ex(q_win, K, Hq, Hkv, L, d, W, pool, 0u, nullptr, scores_out, workspace,
+                        ws_bytes, stream);
 }
 
 sgdkv_status sgdkv_score_static(const void* q_win, const void* K, int32_t Hq, int32_t Hkv,
@@ -213,7 +219,7 @@ sgdkv_status sgdkv_score_static(const void* q_win, const void* K, int32_t Hq, in
   cudaError_t e = cudaMemsetAsync(ws.status, 0, kStatusRegionBytes, st);
   if (e != cudaSuccess) return from_cuda(e);
   e = launch_score(static_cast<const __nv_bfloat16*>(q_win), static_cast<const __nv_bfloat16*>(K),
-                   Hq, Hkv, L, W, pool, 0u, scores_out, ws, st);
+                   Hq, Hkv, L, W, pool, 0u, nullptr, scores_out, ws, st);
   if (e != cudaSuccess) return from_cuda(e);
   if (status_out) {
     e = cudaMemcpyAsync(status_out, ws.status, sizeof(uint32_t), cudaMemcpyDeviceToDevice, st);
@@ -270,7 +276,7 @@ sgdkv_status sgdkv_compress_layer(const void* q_win, const void* K, const void* 
   float* pooled = scores_out ? scores_out : ws.pooled;
   cudaError_t e = launch_score(static_cast<const __nv_bfloat16*>(q_win),
                                static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, pool, 0u,
-                               pooled, ws, st);
+                               nullptr, pooled, ws, st);
   if (e != cudaSuccess) return from_cuda(e);
   return from_cuda(launch_compact(static_cast<const __nv_bfloat16*>(K),
                                   static_cast<const __nv_bfloat16*>(V), pooled, ht, indices_out,

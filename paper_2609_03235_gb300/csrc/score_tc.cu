@@ -67,6 +67,8 @@ struct TcParams {
   int nparts;     // pass 2: partial slots per head written by pass 1
   float scale2;   // log2(e) / sqrt(d)
   int causal;     // 1: window row w sees keys <= L - W + w; 0: every row sees all L keys
+  int agg;        // SGDKV_SCORE_AGG_* >> 1: 0 sum over the group, 1 IPT max, 2 IPT mean, 3 IPT only
+  const float* head_w;   // IPT modes: summarization score per query head [Hq]
   uint64_t wait_ns;
   uint32_t flags;
 };
@@ -625,6 +627,11 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
 // ---------------------------------------------------------------------------------------
 // Pass 2: per key, sum over window rows of 2^(t - lse)
 // ---------------------------------------------------------------------------------------
+// PERG (IPT max aggregation): each epilogue warp takes the 16-column blocks of whole query
+// heads (head g goes to the warps with wi = g % 4, W % 16 == 0, G <= 8), keeps a sum per
+// head and writes the larger of its (at most two) weighted head sums; the four planes are
+// then combined by max instead of sum.
+template <bool PERG>
 __global__ void __maxnreg__(kMaxRegs)
 score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                TcParams p, Ws ws) {
@@ -693,19 +700,43 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
           M = mn;
         }
       }
-      lse2[r] = -(M + log2f(S));                  // stored negated: the bias of the FMA
+      float bias = 0.f;                           // log2 of the row's weight in the sum
+      if (p.agg != 0) {
+        const int G = p.GW / p.W, g = r / p.W;
+        const float* wq = p.head_w + h * G;       // the group's summarization scores
+        auto ok_w = [&](float x) { return x >= 0.f && x < INFINITY; };
+        const float w = wq[g];
+        if (!ok_w(w)) record_error(ws.status, SGDKV_ERR_INVALID_ARG);
+        if (p.agg == 3) {                         // only the group's top head (lower g on ties)
+          int best = 0;
+          float bw = ok_w(wq[0]) ? wq[0] : -1.f;
+          for (int i = 1; i < G; ++i) {
+            const float x = ok_w(wq[i]) ? wq[i] : -1.f;
+            if (x > bw) {
+              bw = x;
+              best = i;
+            }
+          }
+          bias = g == best ? 0.f : -INFINITY;
+        } else {
+          const float x = ok_w(w) ? (p.agg == 2 ? w / float(G) : w) : 0.f;
+          bias = x > 0.f ? log2f(x) : -INFINITY;
+        }
+      }
+      lse2[r] = bias - (M + log2f(S));            // stored negated: the bias of the FMA
     }
     asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
     const uint64_t s22 = pk(p.scale2, p.scale2);
     // The 4 warps of lane quarter q share its 32 keys; the window rows of every N chunk
-    // are dealt to them in blocks of 16 columns, round robin over the whole tile.
+    // are dealt to them in blocks of 16 columns, round robin over the whole tile (PERG: by
+    // query head).
     const int gpc = nn / 16;                     // 16-column blocks per chunk (<= 16)
     float* raw_out = ws.raw + int64_t(wi) * p.Hkv * p.L + int64_t(h) * p.L;
     const int lim_base = p.causal ? int(p.L - p.W) : int(p.L - 1);   // lowest row limit
     bool ok = true;
     for (int n = 0; ok; ++n) {
       int j = 0;
-      uint64_t acc0 = 0, acc1 = 0;
+      uint64_t acc0 = 0, acc1 = 0, acc2 = 0, acc3 = 0;   // PERG: acc0/1 head slot 0, acc2/3 slot 1
       for (int c = 0; c < nch; ++c) {
         const int u = n * nch + c, slot = u & 1;
         if (!(ok = bwait(bar_tfull(s, slot), (u >> 1) & 1, ab, p.wait_ns, ws.status))) break;
@@ -718,13 +749,22 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
         const int key0 = tile * kTileKeys;
         j = key0 + 32 * q + lane;
         const bool masked = key0 + kTileKeys - 1 > lim_base;
-        const int li0 = (((wi - c * gpc) % 4) + 4) % 4;   // first block of this warp in chunk c
-        const int ng = li0 < gpc ? (gpc - li0 + 3) / 4 : 0;
+        // this warp's blocks of chunk c (at most 4)
+        int blk[4], ng = 0;
+        if (PERG) {
+          for (int b = 0; b < gpc && ng < 4; ++b)
+            if (((c * nn + 16 * b) / p.W) % 4 == wi) blk[ng++] = b;
+        } else {
+          const int li0 = (((wi - c * gpc) % 4) + 4) % 4;   // first block of this warp in chunk c
+          ng = li0 < gpc ? (gpc - li0 + 3) / 4 : 0;
+#pragma unroll
+          for (int k = 0; k < 4; ++k) blk[k] = li0 + 4 * k;
+        }
         const uint32_t tb = tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256);
         uint32_t v[4][16];
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          if (k < ng) tmem_ld16(tb + uint32_t((li0 + 4 * k) * 16), v[k]);
+          if (k < ng) tmem_ld16(tb + uint32_t(blk[k] * 16), v[k]);
         tmem_wait_ld();
         tc_fence_before();
         __syncwarp();
@@ -732,22 +772,32 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
           if (k >= ng) continue;
-          const int r0 = c * nn + (li0 + 4 * k) * 16;
+          const int r0 = c * nn + blk[k] * 16;
           if (masked) {                            // rows that cannot see key j drop out
 #pragma unroll
             for (int e = 0; e < 16; ++e)
               if (j > (p.causal ? lim_base + (r0 + e) % p.W : lim_base)) v[k][e] = 0xff800000u;
           }
           const float4* nl = reinterpret_cast<const float4*>(lse2 + r0);
+          const bool second = PERG && (r0 / p.W) >= 4;     // head slot of this block
+          uint64_t a0 = second ? acc2 : acc0, a1 = second ? acc3 : acc1;
 #pragma unroll
           for (int e = 0; e < 16; e += 4) {
             const float4 b = nl[e >> 2];
-            acc0 = acc_exp2(acc0, v[k][e], v[k][e + 1], s22, pk(b.x, b.y));
-            acc1 = acc_exp2(acc1, v[k][e + 2], v[k][e + 3], s22, pk(b.z, b.w));
+            a0 = acc_exp2(a0, v[k][e], v[k][e + 1], s22, pk(b.x, b.y));
+            a1 = acc_exp2(a1, v[k][e + 2], v[k][e + 3], s22, pk(b.z, b.w));
+          }
+          if (second) {
+            acc2 = a0;
+            acc3 = a1;
+          } else {
+            acc0 = a0;
+            acc1 = a1;
           }
         }
       }
-      if (ok && j < p.L) raw_out[j] = hsum(acc0, acc1);
+      if (ok && j < p.L)
+        raw_out[j] = PERG ? fmaxf(hsum(acc0, acc1), hsum(acc2, acc3)) : hsum(acc0, acc1);
     }
   }
   teardown(tmem);
@@ -765,7 +815,7 @@ constexpr int kMaxRadius = 31;                    // pool <= 63
 
 __global__ void __launch_bounds__(kPoolThreads)
 maxpool_sum_kernel(const float* __restrict__ raw, float* __restrict__ out, int64_t L,
-                   int64_t plane, int radius) {
+                   int64_t plane, int radius, int combine_max) {
   __shared__ float sum[kPoolTile + 2 * kMaxRadius];
   const int64_t tiles = ceil_div(L, kPoolTile);
   const int h = int(blockIdx.x / tiles);
@@ -775,9 +825,11 @@ maxpool_sum_kernel(const float* __restrict__ raw, float* __restrict__ out, int64
   for (int i = threadIdx.x; i < span; i += kPoolThreads) {
     const int64_t j = base - radius + i;
     float v = -INFINITY;
-    if (j >= 0 && j < L)
-      v = (__ldcg(r0 + j) + __ldcg(r0 + plane + j)) +
-          (__ldcg(r0 + 2 * plane + j) + __ldcg(r0 + 3 * plane + j));
+    if (j >= 0 && j < L) {
+      const float a = __ldcg(r0 + j), b = __ldcg(r0 + plane + j);
+      const float c = __ldcg(r0 + 2 * plane + j), d = __ldcg(r0 + 3 * plane + j);
+      v = combine_max ? fmaxf(fmaxf(a, b), fmaxf(c, d)) : (a + b) + (c + d);
+    }
     sum[i] = v;
   }
   __syncthreads();
@@ -833,8 +885,8 @@ uint64_t g_score_wait_ns = 2000000000ull;
 uint32_t g_score_flags = 0;
 
 cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
-                         int64_t L, int W, int pool, uint32_t flags, float* scores_out,
-                         const Ws& ws, cudaStream_t stream) {
+                         int64_t L, int W, int pool, uint32_t flags, const float* head_weights,
+                         float* scores_out, const Ws& ws, cudaStream_t stream) {
   if (pool < 1 || pool / 2 > kMaxRadius) return cudaErrorInvalidValue;
   TcParams p{};
   p.Hkv = Hkv;
@@ -852,6 +904,10 @@ cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq,
   if (p.nparts > kMaxScoreParts) return cudaErrorInvalidConfiguration;
   p.scale2 = kLog2e / sqrtf(float(kD));
   p.causal = (flags & SGDKV_SCORE_PROXY_QUERY) ? 0 : 1;
+  p.agg = int((flags & SGDKV_SCORE_AGG_MASK) >> 1);
+  p.head_w = head_weights;
+  if (p.agg != 0 && !head_weights) return cudaErrorInvalidValue;
+  if (p.agg == 1 && (W % 16 != 0 || W > 64 || p.G > 8)) return cudaErrorInvalidValue;
   p.wait_ns = g_score_wait_ns;
   p.flags = g_score_flags;
 
@@ -879,7 +935,9 @@ cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq,
   if ((e = cudaFuncSetAttribute(pass1, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 int(smem1))) != cudaSuccess)
     return e;
-  if ((e = cudaFuncSetAttribute(score_pass2_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  void (*pass2)(const CUtensorMap, const CUtensorMap, TcParams, Ws) =
+      p.agg == 1 ? score_pass2_tc<true> : score_pass2_tc<false>;
+  if ((e = cudaFuncSetAttribute(pass2, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 int(smem2))) != cudaSuccess)
     return e;
   const int grid = Hkv * p.cph;
@@ -889,13 +947,14 @@ cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq,
   }
   {
     KernelTimer t(SGDKV_KERNEL_SCORE_PASS2, stream);
-    score_pass2_tc<<<grid, kThreads, smem2, stream>>>(tm_q, tm_k, p2, ws);
+    pass2<<<grid, kThreads, smem2, stream>>>(tm_q, tm_k, p2, ws);
   }
   {
     KernelTimer t(SGDKV_KERNEL_POOL, stream);
     const unsigned blocks = unsigned(int64_t(Hkv) * ceil_div(L, kPoolTile));
     maxpool_sum_kernel<<<blocks, kPoolThreads, 0, stream>>>(ws.raw, scores_out, L,
-                                                            int64_t(Hkv) * L, pool / 2);
+                                                            int64_t(Hkv) * L, pool / 2,
+                                                            p.agg == 1 ? 1 : 0);
   }
   note_launches(3);
   return cudaGetLastError();

@@ -77,10 +77,11 @@ extern uint64_t g_score_wait_ns;
 extern uint32_t g_score_flags;
 
 // Launchers (each returns cudaGetLastError() after its launches).
-// flags: SGDKV_SCORE_* (0: the causal observation window of sgdkv_score).
+// flags: SGDKV_SCORE_* (0: the causal observation window of sgdkv_score, summed over the
+// GQA group); head_weights: device fp32 [Hq] for the IPT aggregation modes, else NULL.
 cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
-                         int64_t L, int W, int pool, uint32_t flags, float* scores_out,
-                         const Ws& ws, cudaStream_t stream);
+                         int64_t L, int W, int pool, uint32_t flags, const float* head_weights,
+                         float* scores_out, const Ws& ws, cudaStream_t stream);
 cudaError_t launch_compact(const __nv_bfloat16* K, const __nv_bfloat16* V,
                            const float* scores, const HeadTable& ht, int32_t* indices_out,
                            int32_t* cu_out, __nv_bfloat16* K_out, __nv_bfloat16* V_out,

@@ -70,7 +70,7 @@ def lib():
         L.sgdkv_last_cuda_error_string.restype = ctypes.c_char_p
         L.sgdkv_score_ex.restype = ctypes.c_int
         L.sgdkv_score_ex.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, _I32, ctypes.c_uint32,
-                                     _P, _P, _SZ, _P]
+                                     _P, _P, _P, _SZ, _P]
         L.sgdkv_score_static.restype = ctypes.c_int
         L.sgdkv_score_static.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, _I32, _P, _P, _P]
         L.sgdkv_debug_set_score_hooks.restype = None
@@ -133,21 +133,24 @@ def make_workspace(Hq: int, Hkv: int, L: int, W: int, device="cuda", d: int = 12
 
 
 SCORE_PROXY_QUERY = 1
+SCORE_AGG_SUM, SCORE_AGG_IPT_MAX, SCORE_AGG_IPT_MEAN, SCORE_AGG_IPT_ONLY = 0, 2, 4, 6
 
 
-def sgdkv_score(q_win, K, W: int, pool: int, scores_out, workspace, stream=None, flags: int = 0):
-    """Window scores (flags 0: causal observation window) or, with SCORE_PROXY_QUERY,
-    scores of external queries that see every key (sgdkv_score_ex)."""
+def sgdkv_score(q_win, K, W: int, pool: int, scores_out, workspace, stream=None, flags: int = 0,
+                head_weights=None):
+    """Window scores (flags 0: causal observation window, summed over the GQA group) or,
+    through sgdkv_score_ex, SCORE_PROXY_QUERY (external queries that see every key) and the
+    SCORE_AGG_IPT_* group aggregations (head_weights: device fp32 [Hq])."""
     Hq, W_, d = q_win.shape
     Hkv, L, _ = K.shape
-    if flags == 0:
+    if flags == 0 and head_weights is None:
         st = lib().sgdkv_score(_ptr(q_win), _ptr(K), Hq, Hkv, L, d, W, pool, _ptr(scores_out),
                                _ptr(workspace), workspace.numel(), _stream(stream))
         _check(st, "sgdkv_score")
         return
     st = lib().sgdkv_score_ex(_ptr(q_win), _ptr(K), Hq, Hkv, L, d, W, pool, int(flags),
-                              _ptr(scores_out), _ptr(workspace), workspace.numel(),
-                              _stream(stream))
+                              _ptr(head_weights), _ptr(scores_out), _ptr(workspace),
+                              workspace.numel(), _stream(stream))
     _check(st, "sgdkv_score_ex")
 
 

@@ -119,12 +119,20 @@ def test_score_rejects_bad_args_before_device_work():
     assert L.sgdkv_score(p, p, 28, 4, 1024, 128, 32, 6, p, p, 1 << 30, None) == sg.ERR_INVALID_ARG
     # workspace too small
     assert L.sgdkv_score(p, p, 28, 4, 1024, 128, 32, 7, p, p, 16, None) == sg.ERR_WORKSPACE
-    # sgdkv_score_ex: unknown flag bits, then the same checks as sgdkv_score
-    assert L.sgdkv_score_ex(p, p, 28, 4, 1024, 128, 32, 7, 2, p, p, 1 << 30, None) == sg.ERR_INVALID_ARG
-    assert L.sgdkv_score_ex(p, p, 28, 4, 1024, 128, 32, 6, sg.SCORE_PROXY_QUERY, p, p, 1 << 30,
-                            None) == sg.ERR_INVALID_ARG
-    assert L.sgdkv_score_ex(p, p, 28, 4, 1024, 128, 32, 7, sg.SCORE_PROXY_QUERY, p, p, 16,
-                            None) == sg.ERR_WORKSPACE
+    # sgdkv_score_ex: unknown flag bits, an IPT mode without weights, unsupported IPT max
+    # shapes, then the same checks as sgdkv_score
+    ex = L.sgdkv_score_ex
+    assert ex(p, p, 28, 4, 1024, 128, 32, 7, 8, None, p, p, 1 << 30, None) == sg.ERR_INVALID_ARG
+    assert ex(p, p, 28, 4, 1024, 128, 32, 7, sg.SCORE_AGG_IPT_MAX, None, p, p, 1 << 30,
+              None) == sg.ERR_INVALID_ARG
+    assert ex(p, p, 36, 4, 1024, 128, 32, 7, sg.SCORE_AGG_IPT_MAX, p, p, p, 1 << 30,
+              None) == sg.ERR_UNSUPPORTED                              # G = 9 > 8
+    assert ex(p, p, 4, 4, 1024, 128, 96, 7, sg.SCORE_AGG_IPT_MAX, p, p, p, 1 << 30,
+              None) == sg.ERR_UNSUPPORTED                              # W = 96 > 64
+    assert ex(p, p, 28, 4, 1024, 128, 32, 6, sg.SCORE_PROXY_QUERY, None, p, p, 1 << 30,
+              None) == sg.ERR_INVALID_ARG
+    assert ex(p, p, 28, 4, 1024, 128, 32, 7, sg.SCORE_PROXY_QUERY | sg.SCORE_AGG_IPT_MEAN, p, p,
+              p, 16, None) == sg.ERR_WORKSPACE
 
 
 def test_compact_rejects_bad_budgets():

@@ -97,6 +97,62 @@ def test_proxy_query_score_parity(dev, Hq, Hkv, L, W, pool):
         assert np.allclose(got.astype(np.float64).sum(axis=1), Hq // Hkv * W, rtol=1e-4)
 
 
+IPT_SHAPES = [
+    # Hq, Hkv, L, W
+    (14, 2, 1000, 32),     # G*W = 224: one row chunk
+    (28, 4, 3000, 64),     # G*W = 448: two chunks, head 3 split across them
+    (16, 2, 2049, 64),     # G = 8, G*W = 512
+    (4, 4, 700, 32),       # G = 1
+]
+IPT_MODES = [("max", 2, "AGG_IPT_MAX"), ("mean", 4, "AGG_IPT_MEAN"), ("only", 6, "AGG_IPT_ONLY")]
+
+
+def _ipt_weights(Hq, seed):
+    w = np.random.default_rng(seed).random(Hq).astype(np.float32)
+    w[0] = 0.0                              # a head that contributes nothing
+    if Hq > 3:
+        w[3] = w[2]                         # a tie (Ipt only: lower head wins)
+    return w
+
+
+@pytest.mark.parametrize("Hq,Hkv,L,W", IPT_SHAPES)
+@pytest.mark.parametrize("mode", IPT_MODES, ids=[m[0] for m in IPT_MODES])
+@pytest.mark.parametrize("proxy", [False, True])
+def test_ipt_aggregation_parity(dev, Hq, Hkv, L, W, mode, proxy):
+    """Summarization-weighted GQA aggregation against the oracle (appendix variants)."""
+    name, flag, omode = mode
+    wl = synth.tiny_workload(Hq=Hq, Hkv=Hkv, d=128, L=L, W=W, n_salient=min(8, max(0, L - W - 4)))
+    inp = synth.tiny_inputs(wl, tag=700 + L)
+    q, K, _ = _upload(inp, dev)
+    w = _ipt_weights(Hq, L)
+    ws = sg.make_workspace(Hq, Hkv, L, W, dev)
+    out = torch.empty((Hkv, L), dtype=torch.float32, device=dev)
+    flags = flag | (sg.SCORE_PROXY_QUERY if proxy else 0)
+    sg.sgdkv_score(q, K, W, 7, out, ws, flags=flags, head_weights=torch.from_numpy(w).to(dev))
+    torch.cuda.synchronize()
+    assert sg.sgdkv_last_error(ws) == sg.OK
+    raw = O.window_scores_ipt(inp["q"], inp["K"], w, getattr(O, omode), causal=not proxy)
+    exp = O.max_pool(raw, 7)
+    got = out.cpu().numpy()
+    ok = _within(got, exp)
+    assert ok.all(), f"{(~ok).sum()} of {ok.size} off; worst {np.max(np.abs(got - exp))}"
+
+
+def test_ipt_negative_weight_is_reported(dev):
+    wl = synth.tiny_workload(Hq=14, Hkv=2, d=128, L=500, W=32, n_salient=4)
+    inp = synth.tiny_inputs(wl, tag=799)
+    q, K, _ = _upload(inp, dev)
+    w = np.ones(14, np.float32)
+    w[5] = -1.0
+    ws = sg.make_workspace(14, 2, 500, 32, dev)
+    out = torch.empty((2, 500), dtype=torch.float32, device=dev)
+    sg.sgdkv_score(q, K, 32, 7, out, ws, flags=sg.SCORE_AGG_IPT_MEAN,
+                   head_weights=torch.from_numpy(w).to(dev))
+    torch.cuda.synchronize()
+    assert sg.sgdkv_last_error(ws) == sg.ERR_INVALID_ARG
+    assert sg.sgdkv_last_error(ws) == sg.OK                   # reading clears it
+
+
 def _tie_heavy_scores(rng, Hkv, L):
     return (rng.integers(0, 6, size=(Hkv, L)) * 0.125).astype(np.float32)
 

@@ -156,3 +156,59 @@ def test_max_pool_spike_plateau():
 def test_max_pool_rejects_even_kernel():
     with pytest.raises(ValueError):
         O.max_pool(np.zeros((1, 4), np.float32), 4)
+
+
+# -- summarization-weighted GQA aggregation ("Ipt." variants of the appendix) --------------
+
+def _ipt_case(seed, Hq=6, Hkv=2, L=40, W=8, d=16):
+    rng = np.random.default_rng(seed)
+    return rng.standard_normal((Hq, W, d)), rng.standard_normal((Hkv, L, d)) * 2
+
+
+def test_ipt_head_attention_sums_to_window_scores():
+    """Summing the per-head attention over a group gives window_scores (no weights)."""
+    q, k = _ipt_case(1)
+    A = O.head_window_attention(q, k)
+    raw = O.window_scores(q, k).astype(np.float64)
+    assert np.allclose(A.reshape(2, 3, -1).sum(axis=1), raw, rtol=1e-6)
+    assert np.allclose(A.sum(axis=1), q.shape[1], rtol=1e-9)       # each head: W rows of 1
+
+
+def test_ipt_modes_on_identical_heads():
+    """Every query head of a group equal: max of w_g A = max(w) A, mean = mean(w) A, only = A."""
+    q, k = _ipt_case(2, Hq=3, Hkv=1)
+    q[1] = q[0]
+    q[2] = q[0]
+    w = np.array([0.2, 0.9, 0.5])
+    A = O.head_window_attention(q, k)[0]
+    assert np.allclose(O.window_scores_ipt(q, k, w, O.AGG_IPT_MAX), 0.9 * A, rtol=1e-6)
+    assert np.allclose(O.window_scores_ipt(q, k, w, O.AGG_IPT_MEAN), w.mean() * A, rtol=1e-6)
+    assert np.allclose(O.window_scores_ipt(q, k, w, O.AGG_IPT_ONLY), A, rtol=1e-6)
+
+
+def test_ipt_only_picks_the_top_head_lower_index_on_ties():
+    q, k = _ipt_case(3, Hq=4, Hkv=1)
+    A = O.head_window_attention(q, k)
+    assert np.allclose(O.window_scores_ipt(q, k, [0.1, 0.7, 0.7, 0.2], O.AGG_IPT_ONLY)[0],
+                       A[1], rtol=1e-6)
+
+
+def test_ipt_max_takes_the_larger_weighted_head_per_key():
+    """Brute force on a tiny case: the weighted maximum per key, and zero weights drop heads."""
+    q, k = _ipt_case(4, Hq=4, Hkv=2, L=25)
+    w = np.array([0.5, 0.0, 2.0, 1.0])
+    A = O.head_window_attention(q, k)
+    got = O.window_scores_ipt(q, k, w, O.AGG_IPT_MAX).astype(np.float64)
+    for h in range(2):
+        for j in range(25):
+            assert np.isclose(got[h, j], max(w[2 * h] * A[2 * h, j], w[2 * h + 1] * A[2 * h + 1, j]),
+                              rtol=1e-6)
+    assert np.allclose(got[0], 0.5 * A[0], rtol=1e-6)              # head 1 has weight 0
+
+
+def test_ipt_rejects_bad_weights():
+    q, k = _ipt_case(5)
+    with pytest.raises(ValueError):
+        O.window_scores_ipt(q, k, [1, 1, 1, 1, 1, -1], O.AGG_IPT_MAX)
+    with pytest.raises(ValueError):
+        O.window_scores_ipt(q, k, [1, 1, 1], O.AGG_IPT_MAX)
