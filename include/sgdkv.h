@@ -189,7 +189,10 @@ SGDKV_API sgdkv_status sgdkv_score_static(const void* q_win, const void* K, int3
  * [L - n_recent, L), plus the (b_h - n_sink - n_recent) middle positions with the highest
  * scores (equal scores: lower position first).  Kept positions are written ascending.
  *
- * K, V            device bf16 [Hkv][L][d]
+ * K, V            bf16 [Hkv][L][d]: device memory, or pinned host memory that the device
+ *                 addresses directly (cudaHostAlloc, cudaHostRegister).  Only the kept rows
+ *                 are read (by the gather), so a cache held in host memory crosses the host
+ *                 link for the kept rows alone.
  * scores          device fp32 [Hkv][L], finite and >= 0 (as produced by sgdkv_score)
  * budgets         HOST int64 [Hkv], n_sink + n_recent <= b_h <= L
  * indices_out     device int32 [sum b_h]: kept positions, head by head
@@ -206,7 +209,9 @@ SGDKV_API sgdkv_status sgdkv_compact(const void* K, const void* V, const float* 
 /*
  * The whole per-layer step: sgdkv_score followed by sgdkv_compact on the same stream,
  * keeping the pooled scores in the workspace.  scores_out may be NULL; when given, it
- * receives the pooled scores as sgdkv_score would.  Other arguments as above.
+ * receives the pooled scores as sgdkv_score would.  K must be device memory (the scorer
+ * streams it with TMA); V may be pinned host memory as in sgdkv_compact.  Other arguments
+ * as above.
  */
 SGDKV_API sgdkv_status sgdkv_compress_layer(const void* q_win, const void* K, const void* V,
                                   const int64_t* budgets, int32_t Hq, int32_t Hkv, int64_t L,

@@ -326,3 +326,43 @@ def test_layers_on_two_streams(dev):
     for (inp, q, K, V, ws, s), out in zip(runs, outs):
         assert sg.sgdkv_last_error(ws) == sg.OK
         _check_end_to_end(inp, out, b, 128, 128, 7)
+
+
+def test_compact_reads_kv_from_pinned_host_memory(dev):
+    """K and V of sgdkv_compact (and V of sgdkv_compress_layer) may be pinned host memory:
+    the gather reads the kept rows across the host link; outputs bit-exact."""
+    rng = np.random.default_rng(11)
+    Hkv, L = 3, 3000
+    scores = rng.random((Hkv, L)).astype(np.float32)
+    K = synth.bf16_round(rng.standard_normal((Hkv, L, 128), dtype=np.float32))
+    V = synth.bf16_round(rng.standard_normal((Hkv, L, 128), dtype=np.float32))
+    b = np.array([700, 64, 3000], np.int64)
+    total = int(b.sum())
+    Kh = synth.to_torch_bf16(K, "cpu").pin_memory()
+    Vh = synth.to_torch_bf16(V, "cpu").pin_memory()
+    ws = sg.make_workspace(Hkv, Hkv, L, 32, dev)
+    st = torch.from_numpy(scores).to(dev)
+    idx = torch.empty(total, dtype=torch.int32, device=dev)
+    cu = torch.empty(Hkv + 1, dtype=torch.int32, device=dev)
+    ko = torch.empty((total, 128), dtype=torch.bfloat16, device=dev)
+    vo = torch.empty((total, 128), dtype=torch.bfloat16, device=dev)
+    sg.sgdkv_compact(Kh, Vh, st, b, 16, 16, idx, cu, ko, vo, ws)
+    torch.cuda.synchronize()
+    assert sg.sgdkv_last_error(ws) == sg.OK
+    e_idx, e_cu = O.select_indices(scores, b, 16, 16)
+    assert np.array_equal(idx.cpu().numpy(), e_idx)
+    e_ko, e_vo = O.gather(K, V, e_idx, e_cu)
+    assert np.array_equal(synth.from_torch_bf16(ko), e_ko)
+    assert np.array_equal(synth.from_torch_bf16(vo), e_vo)
+
+    # compress_layer: K on the device, V in pinned host memory
+    wl = synth.tiny_workload(Hq=28, Hkv=4, d=128, L=5000, W=64, n_salient=32, floor=256)
+    inp = synth.tiny_inputs(wl, tag=301)
+    q, Kd, _ = _upload(inp, dev)
+    Vh = synth.to_torch_bf16(inp["V"], "cpu").pin_memory()
+    b = np.array([1250, 700, 2400, 256], np.int64)
+    ws = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
+    out = sg.compress_layer_alloc(q, Kd, Vh, b, wl.W, 7, 128, 128, ws)
+    torch.cuda.synchronize()
+    assert sg.sgdkv_last_error(ws) == sg.OK
+    _check_end_to_end(inp, out, b, 128, 128, 7)
