@@ -749,22 +749,20 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
         const int key0 = tile * kTileKeys;
         j = key0 + 32 * q + lane;
         const bool masked = key0 + kTileKeys - 1 > lim_base;
-        // this warp's blocks of chunk c (at most 4)
-        int blk[4], ng = 0;
+        // this warp's blocks of chunk c (at most 4): block k is li0 + 4k (PERG: blk[k])
+        int blk[4], ng = 0, li0 = 0;
         if (PERG) {
           for (int b = 0; b < gpc && ng < 4; ++b)
             if (((c * nn + 16 * b) / p.W) % 4 == wi) blk[ng++] = b;
         } else {
-          const int li0 = (((wi - c * gpc) % 4) + 4) % 4;   // first block of this warp in chunk c
+          li0 = (((wi - c * gpc) % 4) + 4) % 4;   // first block of this warp in chunk c
           ng = li0 < gpc ? (gpc - li0 + 3) / 4 : 0;
-#pragma unroll
-          for (int k = 0; k < 4; ++k) blk[k] = li0 + 4 * k;
         }
         const uint32_t tb = tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256);
         uint32_t v[4][16];
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          if (k < ng) tmem_ld16(tb + uint32_t(blk[k] * 16), v[k]);
+          if (k < ng) tmem_ld16(tb + uint32_t((PERG ? blk[k] : li0 + 4 * k) * 16), v[k]);
         tmem_wait_ld();
         tc_fence_before();
         __syncwarp();
@@ -772,7 +770,7 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
           if (k >= ng) continue;
-          const int r0 = c * nn + blk[k] * 16;
+          const int r0 = c * nn + (PERG ? blk[k] : li0 + 4 * k) * 16;
           if (masked) {                            // rows that cannot see key j drop out
 #pragma unroll
             for (int e = 0; e < 16; ++e)
