@@ -232,6 +232,22 @@ def path_bytes(wl, budgets_layer) -> float:
 # our arm
 # ------------------------------------------------------------------------------------------
 
+def workload_config(wl, args, world, n_layers):
+    """The `config` object of both arms' JSON lines (the same workload for both)."""
+    from paper_2609_03235_gb300 import configs
+    n_sink, n_recent = configs.sink_recent_split(wl.floor)
+    return {"workload": wl.name, "model_shape": "Qwen2.5-7B-1M" if wl.Hkv == 4 else "Qwen3-32B",
+            "n_layers": n_layers, "Hq": wl.Hq, "Hkv": wl.Hkv, "head_dim": wl.d,
+            "context_len": wl.L, "window": wl.W, "pool": wl.pool,
+            "budget_frac": args.frac, "floor": wl.floor, "n_sink": n_sink,
+            "n_recent": n_recent, "parallelism": f"replicas x{world}",
+            "streams": "scoring on one stream, selection + gather on a second; layer "
+                       "l's compaction overlaps layer l+1's scoring",
+            "l2": "inputs larger than L2 (K+V of one layer = %d MiB)" %
+                  (2 * wl.Hkv * wl.L * wl.d * 2 >> 20)}
+
+
+
 def run_ours(args, world, rank, local):
     import numpy as np
     import torch
@@ -362,15 +378,7 @@ def run_ours(args, world, rank, local):
         "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded N(0,1) K/V/Q with planted sink and salient keys)",
-        "config": {"workload": wl.name, "model_shape": "Qwen2.5-7B-1M" if wl.Hkv == 4 else "Qwen3-32B",
-                   "n_layers": Ls, "Hq": wl.Hq, "Hkv": wl.Hkv, "head_dim": wl.d,
-                   "context_len": wl.L, "window": wl.W, "pool": wl.pool,
-                   "budget_frac": args.frac, "floor": wl.floor, "n_sink": n_sink,
-                   "n_recent": n_recent, "parallelism": f"replicas x{world}",
-                   "streams": "scoring on one stream, selection + gather on a second; layer "
-                              "l's compaction overlaps layer l+1's scoring",
-                   "l2": "inputs larger than L2 (K+V of one layer = %d MiB)" %
-                         (2 * wl.Hkv * wl.L * wl.d * 2 >> 20)},
+        "config": workload_config(wl, args, world, Ls),
         "roofline": {"kernel": top, "bound": "tensor", "achieved": achieved_tf,
                      "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
                      "frac": achieved_tf / peaks["bf16_sus"],
@@ -556,7 +564,8 @@ def run_reference(args, world, rank):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded, host-generated)", "impl": "reference",
-            "config": {"workload": wl.name, "budget_frac": args.frac},
+            "config": workload_config(wl, args, world,
+                                      wl.n_layers if args.layers <= 0 else min(args.layers, wl.n_layers)),
             "cpu_baseline": {"value": value, "unit": UNIT, "kind": "oracle", "cores": cores,
                              "sample": f"each step: 1 KV head of 1 layer of {wl.name}"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
