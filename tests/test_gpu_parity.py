@@ -366,3 +366,43 @@ def test_compact_reads_kv_from_pinned_host_memory(dev):
     torch.cuda.synchronize()
     assert sg.sgdkv_last_error(ws) == sg.OK
     _check_end_to_end(inp, out, b, 128, 128, 7)
+
+
+def test_bench_launch_configuration_full_size(dev):
+    """The schedule bench.py times, at full size: consecutive layers of the 128K-context
+    Qwen2.5-7B workload, scoring on one stream and selection + gather on a second
+    (separate workspaces, layer l's compaction overlapping layer l+1's scoring); every
+    layer end to end against the oracle."""
+    wl = configs.BY_NAME["c3_qwen25_7b_L128k"]
+    n_sink, n_recent = configs.sink_recent_split(wl.floor)
+    all_b = sg.sgdkv_allocate_budgets(synth.head_scores(wl), wl.L, wl.total_budget(0.25), wl.floor)
+    layers = [0, wl.n_layers - 1]
+    ws_a = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
+    ws_b = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
+    stream_a = torch.cuda.current_stream(dev)
+    stream_b = torch.cuda.Stream(dev)
+    runs = []
+    for layer in layers:
+        inp = synth.layer_inputs_host(wl, layer)
+        q, K, V = _upload(inp, dev)
+        b = all_b[layer * wl.Hkv:(layer + 1) * wl.Hkv]
+        tot = int(b.sum())
+        out = dict(scores=torch.empty((wl.Hkv, wl.L), dtype=torch.float32, device=dev),
+                   indices=torch.empty(tot, dtype=torch.int32, device=dev),
+                   cu_seqlens=torch.empty(wl.Hkv + 1, dtype=torch.int32, device=dev),
+                   K_out=torch.empty((tot, wl.d), dtype=torch.bfloat16, device=dev),
+                   V_out=torch.empty((tot, wl.d), dtype=torch.bfloat16, device=dev))
+        runs.append((inp, q, K, V, b, out))
+    torch.cuda.synchronize()
+    for inp, q, K, V, b, out in runs:
+        sg.sgdkv_score(q, K, wl.W, wl.pool, out["scores"], ws_a, stream_a)
+        ev = torch.cuda.Event()
+        ev.record(stream_a)
+        stream_b.wait_event(ev)
+        sg.sgdkv_compact(K, V, out["scores"], b, n_sink, n_recent, out["indices"],
+                         out["cu_seqlens"], out["K_out"], out["V_out"], ws_b, stream_b)
+    torch.cuda.synchronize()
+    assert sg.sgdkv_last_error(ws_a) == sg.OK
+    assert sg.sgdkv_last_error(ws_b) == sg.OK
+    for inp, q, K, V, b, out in runs:
+        _check_end_to_end(inp, out, b, n_sink, n_recent, wl.pool)
