@@ -222,8 +222,9 @@ SGDKV_API sgdkv_status sgdkv_compress_layer(const void* q_win, const void* K, co
 
 /*
  * Diagnostics: number of kernel launches this process has issued through libsgdkv so far
- * (all entry points, all devices).  No counterpart in the paper; used to report how many
- * of the library's kernels a timed region ran.
+ * (all entry points, all devices).  A launch issued into a stream that is being captured
+ * into a CUDA graph counts once, at capture.  No counterpart in the paper; used to report how
+ * many of the library's kernels a timed region ran.
  */
 SGDKV_API uint64_t sgdkv_launch_count(void);
 
@@ -238,8 +239,11 @@ SGDKV_API const char* sgdkv_last_cuda_error_string(void);
  * the library launches is bracketed by CUDA events on its launch stream (mask 0 turns timing
  * off; each bracket adds two event records to the stream).  sgdkv_debug_kernel_timing synchronises
  * the recorded events of one kernel kind, returns their summed duration in milliseconds and
- * their count, and forgets them.  No counterpart in the paper; used by the benchmark to
- * time its dominant kernel inside the timed region.  Errors: INVALID_ARG, CUDA.
+ * their count, and forgets them.  A launch issued while its stream is being captured into a
+ * CUDA graph is bracketed by event-record nodes of that graph: its record is read after the
+ * graph has been launched (the last launch of the graph), and a graph that has not been
+ * launched yet makes the call fail with CUDA.  No counterpart in the paper; used by the
+ * benchmark to time its dominant kernel inside the timed region.  Errors: INVALID_ARG, CUDA.
  */
 #define SGDKV_KERNEL_SCORE_PASS1 0   /* window logits, per-row max and sum  */
 #define SGDKV_KERNEL_SCORE_PASS2 1   /* per-key sum of normalised weights   */

@@ -86,6 +86,17 @@ __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
                : "memory");
 }
+__device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[32]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
+                 "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
+                 "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]),
+                 "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]),
+                 "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]),
+                 "+r"(r[30]), "+r"(r[31])
+               :
+               : "memory");
+}
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
@@ -239,6 +250,16 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
 }
 __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+// The same wait, with the registers of the load it completes passed through it: code that
+// reads them cannot be scheduled above the wait while a later load is still in flight.
+__device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
+                 "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
+                 "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15])
+               :
+               : "memory");
 }
 __device__ __forceinline__ float ex2(float x) {
   float y;
@@ -581,17 +602,26 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
         const bool edge = kb + 31 > lim_base;
         uint32_t v[2][32];
         const uint32_t tb = tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256 + wi * 32);
-#pragma unroll
-        for (int i = 0; i < 2; ++i)
-          if (2 * g + i < NRT && valid[2 * g + i]) tmem_ld32(tb + uint32_t(i * kTileKeys), v[i]);
-        tmem_wait_ld();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar_tempty(s, slot));   // slot free: data is in registers
-#pragma unroll
-        for (int i = 0; i < 2; ++i) {
-          const int rt = 2 * g + i;
-          if (rt < NRT && valid[rt]) online_fold<32>(v[i], kb, edge, lim[rt], p.scale2, m[rt], Z[rt]);
+        // The second row tile's load is in flight while the first is folded; the slot is
+        // released once both have landed.
+        const int rt0 = 2 * g, rt1 = 2 * g + 1;
+        const bool h0 = rt0 < NRT && valid[rt0], h1 = rt1 < NRT && valid[rt1];
+        if (h0) {
+          tmem_ld32(tb, v[0]);
+          tmem_wait_ld(v[0]);
+        }
+        if (h1) tmem_ld32(tb + uint32_t(kTileKeys), v[1]);
+        auto release = [&] {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar_tempty(s, slot));
+        };
+        if (!h1) release();
+        if (h0) online_fold<32>(v[0], kb, edge, lim[rt0], p.scale2, m[rt0], Z[rt0]);
+        if (h1) {
+          tmem_wait_ld(v[1]);
+          release();
+          online_fold<32>(v[1], kb, edge, lim[rt1], p.scale2, m[rt1], Z[rt1]);
         }
       }
     }
@@ -759,22 +789,30 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
           ng = li0 < gpc ? (gpc - li0 + 3) / 4 : 0;
         }
         const uint32_t tb = tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256);
-        uint32_t v[4][16];
-#pragma unroll
-        for (int k = 0; k < 4; ++k)
-          if (k < ng) tmem_ld16(tb + uint32_t((PERG ? blk[k] : li0 + 4 * k) * 16), v[k]);
-        tmem_wait_ld();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar_tempty(s, slot));   // slot free: data is in registers
+        auto col = [&](int k) { return PERG ? blk[k] : li0 + 4 * k; };
+        // Block k + 1 is loaded while block k is summed; the slot is released as soon as
+        // the last block's load has landed.
+        uint32_t v[2][16];
+        if (ng > 0) {
+          tmem_ld16(tb + uint32_t(col(0) * 16), v[0]);
+          tmem_wait_ld(v[0]);
+        }
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-          if (k >= ng) continue;
-          const int r0 = c * nn + (PERG ? blk[k] : li0 + 4 * k) * 16;
+          if (k >= ng) break;
+          if (k + 1 < ng) {
+            tmem_ld16(tb + uint32_t(col(k + 1) * 16), v[(k + 1) & 1]);
+          } else {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_tempty(s, slot));   // slot free: all of it loaded
+          }
+          uint32_t (&vk)[16] = v[k & 1];
+          const int r0 = c * nn + col(k) * 16;
           if (masked) {                            // rows that cannot see key j drop out
 #pragma unroll
             for (int e = 0; e < 16; ++e)
-              if (j > (p.causal ? lim_base + (r0 + e) % p.W : lim_base)) v[k][e] = 0xff800000u;
+              if (j > (p.causal ? lim_base + (r0 + e) % p.W : lim_base)) vk[e] = 0xff800000u;
           }
           const float4* nl = reinterpret_cast<const float4*>(lse2 + r0);
           const bool second = PERG && (r0 / p.W) >= 4;     // head slot of this block
@@ -782,8 +820,8 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
 #pragma unroll
           for (int e = 0; e < 16; e += 4) {
             const float4 b = nl[e >> 2];
-            a0 = acc_exp2(a0, v[k][e], v[k][e + 1], s22, pk(b.x, b.y));
-            a1 = acc_exp2(a1, v[k][e + 2], v[k][e + 3], s22, pk(b.z, b.w));
+            a0 = acc_exp2(a0, vk[e], vk[e + 1], s22, pk(b.x, b.y));
+            a1 = acc_exp2(a1, vk[e + 2], vk[e + 3], s22, pk(b.z, b.w));
           }
           if (second) {
             acc2 = a0;
@@ -792,6 +830,12 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
             acc0 = a0;
             acc1 = a1;
           }
+          if (k + 1 < ng) tmem_wait_ld(v[(k + 1) & 1]);
+        }
+        if (ng == 0) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar_tempty(s, slot));
         }
       }
       if (ok && j < p.L)

@@ -1,5 +1,7 @@
 // Optional per-kernel timing (diagnostics): CUDA events recorded around every kernel the
-// library launches, on the launch stream, while timing is enabled.
+// library launches, on the launch stream, while timing is enabled.  Launches captured into a
+// CUDA graph are bracketed by event-record nodes of that graph; their records are read after
+// the graph has run (one record per captured launch).
 #include <mutex>
 #include <vector>
 
@@ -26,13 +28,22 @@ cudaEvent_t take_event() {
   if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
   return e;
 }
+
+// Records e on the stream; while the stream is being captured into a CUDA graph the record
+// becomes an event-record node of the graph (taken each time the graph is launched).
+void record(cudaEvent_t e, cudaStream_t stream) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  cudaStreamIsCapturing(stream, &cs);
+  if (cs == cudaStreamCaptureStatusActive) cudaEventRecordWithFlags(e, stream, cudaEventRecordExternal);
+  else cudaEventRecord(e, stream);
+}
 }  // namespace
 
 KernelTimer::KernelTimer(int kind, cudaStream_t stream) : kind_(kind), stream_(stream) {
   std::lock_guard<std::mutex> lock(g_mu);
   if (kind_ < 0 || kind_ >= SGDKV_KERNEL_KINDS || !(g_mask & (1u << kind_))) return;
   start_ = take_event();
-  if (start_) cudaEventRecord(static_cast<cudaEvent_t>(start_), stream_);
+  if (start_) record(static_cast<cudaEvent_t>(start_), stream_);
 }
 
 KernelTimer::~KernelTimer() {
@@ -43,7 +54,7 @@ KernelTimer::~KernelTimer() {
     g_free.push_back(static_cast<cudaEvent_t>(start_));
     return;
   }
-  cudaEventRecord(end, stream_);
+  record(end, stream_);
   g_pending.push_back(Record{kind_, static_cast<cudaEvent_t>(start_), end});
 }
 

@@ -368,10 +368,12 @@ def test_compact_reads_kv_from_pinned_host_memory(dev):
     _check_end_to_end(inp, out, b, 128, 128, 7)
 
 
-def test_bench_launch_configuration_full_size(dev):
+@pytest.mark.parametrize("graph", [False, True])
+def test_bench_launch_configuration_full_size(dev, graph):
     """The schedule bench.py times, at full size: consecutive layers of the 128K-context
     Qwen2.5-7B workload, scoring on one stream and selection + gather on a second
-    (separate workspaces, layer l's compaction overlapping layer l+1's scoring); every
+    (separate workspaces, layer l's compaction overlapping layer l+1's scoring), launched
+    directly or captured into a CUDA graph and replayed (bench.py's timed steps); every
     layer end to end against the oracle."""
     wl = configs.BY_NAME["c3_qwen25_7b_L128k"]
     n_sink, n_recent = configs.sink_recent_split(wl.floor)
@@ -394,13 +396,37 @@ def test_bench_launch_configuration_full_size(dev):
                    V_out=torch.empty((tot, wl.d), dtype=torch.bfloat16, device=dev))
         runs.append((inp, q, K, V, b, out))
     torch.cuda.synchronize()
-    for inp, q, K, V, b, out in runs:
-        sg.sgdkv_score(q, K, wl.W, wl.pool, out["scores"], ws_a, stream_a)
-        ev = torch.cuda.Event()
-        ev.record(stream_a)
-        stream_b.wait_event(ev)
-        sg.sgdkv_compact(K, V, out["scores"], b, n_sink, n_recent, out["indices"],
-                         out["cu_seqlens"], out["K_out"], out["V_out"], ws_b, stream_b)
+
+    def launches(sa):
+        fork = torch.cuda.Event()
+        fork.record(sa)
+        stream_b.wait_event(fork)
+        for inp, q, K, V, b, out in runs:
+            sg.sgdkv_score(q, K, wl.W, wl.pool, out["scores"], ws_a, sa)
+            ev = torch.cuda.Event()
+            ev.record(sa)
+            stream_b.wait_event(ev)
+            sg.sgdkv_compact(K, V, out["scores"], b, n_sink, n_recent, out["indices"],
+                             out["cu_seqlens"], out["K_out"], out["V_out"], ws_b, stream_b)
+        done = torch.cuda.Event()
+        done.record(stream_b)
+        sa.wait_event(done)
+
+    if graph:
+        launches(stream_a)                       # first-use setup outside the capture
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            launches(torch.cuda.current_stream(dev))
+        for inp, q, K, V, b, out in runs:        # the replay must write every output again
+            out["scores"].fill_(float("nan"))
+            out["indices"].fill_(-1)
+            out["cu_seqlens"].fill_(-1)
+            out["K_out"].zero_()
+            out["V_out"].zero_()
+        g.replay()
+    else:
+        launches(stream_a)
     torch.cuda.synchronize()
     assert sg.sgdkv_last_error(ws_a) == sg.OK
     assert sg.sgdkv_last_error(ws_b) == sg.OK
