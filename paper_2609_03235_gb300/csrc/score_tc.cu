@@ -657,6 +657,36 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
 // ---------------------------------------------------------------------------------------
 // Pass 2: per key, sum over window rows of 2^(t - lse)
 // ---------------------------------------------------------------------------------------
+// One pass-2 slot use in the usual case: no key of the tile is masked and the warp's NB
+// blocks of 16 columns sit at li0, li0 + 4, ... (all offsets but li0 fixed at compile time,
+// so the loop has no branches).  Block k + 1 is loaded while block k is summed; the slot is
+// released once the last block has landed.
+template <int NB>
+__device__ __forceinline__ void p2_use(uint32_t tb, int li0, const float* lse_c, uint64_t s22,
+                                       uint32_t tempty, int lane, uint64_t& a0, uint64_t& a1) {
+  uint32_t v[2][16];
+  tmem_ld16(tb + uint32_t(li0 * 16), v[0]);
+  tmem_wait_ld(v[0]);
+#pragma unroll
+  for (int k = 0; k < NB; ++k) {
+    if (k + 1 < NB) {
+      tmem_ld16(tb + uint32_t((li0 + 4 * (k + 1)) * 16), v[(k + 1) & 1]);
+    } else {
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty);
+    }
+    const float4* nl = reinterpret_cast<const float4*>(lse_c + (li0 + 4 * k) * 16);
+#pragma unroll
+    for (int e = 0; e < 16; e += 4) {
+      const float4 b = nl[e >> 2];
+      a0 = acc_exp2(a0, v[k & 1][e], v[k & 1][e + 1], s22, pk(b.x, b.y));
+      a1 = acc_exp2(a1, v[k & 1][e + 2], v[k & 1][e + 3], s22, pk(b.z, b.w));
+    }
+    if (k + 1 < NB) tmem_wait_ld(v[(k + 1) & 1]);
+  }
+}
+
 // PERG (IPT max aggregation): each epilogue warp takes the 16-column blocks of whole query
 // heads (head g goes to the warps with wi = g % 4, W % 16 == 0, G <= 8), keeps a sum per
 // head and writes the larger of its (at most two) weighted head sums; the four planes are
@@ -789,6 +819,16 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
           ng = li0 < gpc ? (gpc - li0 + 3) / 4 : 0;
         }
         const uint32_t tb = tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256);
+        if (!PERG && !masked && ng > 0) {
+          const uint32_t te = bar_tempty(s, slot);
+          const float* lse_c = lse2 + c * nn;
+          if (ng == 4) p2_use<4>(tb, li0, lse_c, s22, te, lane, acc0, acc1);
+          else if (ng == 3) p2_use<3>(tb, li0, lse_c, s22, te, lane, acc0, acc1);
+          else if (ng == 2) p2_use<2>(tb, li0, lse_c, s22, te, lane, acc0, acc1);
+          else p2_use<1>(tb, li0, lse_c, s22, te, lane, acc0, acc1);
+          continue;
+        }
+        // General case: masked keys (the last tiles), blocks by query head (PERG).
         auto col = [&](int k) { return PERG ? blk[k] : li0 + 4 * k; };
         // Block k + 1 is loaded while block k is summed; the slot is released as soon as
         // the last block's load has landed.
