@@ -192,19 +192,19 @@ KERNEL_NAMES = ("score_pass1_tc", "score_pass2_tc", "maxpool_sum_kernel", "sel_c
 # DRAM traffic per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one ncu capture
 # of the 128K-context Qwen2.5-7B layer (28 query / 4 KV heads, W=64), keyed by the SHA-256 of
 # the kernel source it was taken on; a source that has changed since reads as null.
-_SCORE_SHA = "2f306c1957b9d0f6dcbc067270669776f7755ab7d607d37639b8612196f5b699"
+_SCORE_SHA = "bf6ad59d9cc8036492c8592179ed3c4383e93423d2d99f2dda6040bd9bcca892"
 _SELECT_SHA = "390cce311b1188274ecd3021b148b6bbb18954a7a16521c4cd5ba007a67c1d4a"
 MEASURED_TRAFFIC = {
     ("score_pass1_tc", "c3_qwen25_7b_L128k"):
-        {"bytes": 134762752 + 4677376, "source": "score_tc.cu", "sha256": _SCORE_SHA},
+        {"bytes": 134758400 + 4730368, "source": "score_tc.cu", "sha256": _SCORE_SHA},
     ("score_pass2_tc", "c3_qwen25_7b_L128k"):
-        {"bytes": 135463680 + 6326528, "source": "score_tc.cu", "sha256": _SCORE_SHA},
+        {"bytes": 135324416 + 5552128, "source": "score_tc.cu", "sha256": _SCORE_SHA},
     ("maxpool_sum_kernel", "c3_qwen25_7b_L128k"):
-        {"bytes": 8397568 + 0, "source": "score_tc.cu", "sha256": _SCORE_SHA},
+        {"bytes": 8398080 + 0, "source": "score_tc.cu", "sha256": _SCORE_SHA},
     ("sel_cluster_kernel", "c3_qwen25_7b_L128k"):
-        {"bytes": 2144512 + 0, "source": "select.cu", "sha256": _SELECT_SHA},
+        {"bytes": 2144768 + 0, "source": "select.cu", "sha256": _SELECT_SHA},
     ("gather_kernel", "c3_qwen25_7b_L128k"):
-        {"bytes": 40768256 + 1915392, "source": "select.cu", "sha256": _SELECT_SHA},
+        {"bytes": 40769024 + 1928192, "source": "select.cu", "sha256": _SELECT_SHA},
 }
 
 

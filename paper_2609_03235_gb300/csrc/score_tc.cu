@@ -20,9 +20,10 @@
 // through a ring of shared-memory stages); warp 3 allocates the 512 TMEM columns and its
 // elected lane issues the MMAs; warps 4..19 are the epilogue (four per TMEM lane quarter);
 // warps 0 and 1 idle, so that the control warps share sub-partitions with the lane
-// quarters that carry less epilogue work.  An epilogue warp loads all its TMEM columns of a
-// slot, releases the slot, then does the arithmetic, so the MMAs of the next slot overlap
-// it.  Each CTA owns one KV head and claims its key tiles from a counter shared by the
+// quarters that carry less epilogue work.  An epilogue warp loads its TMEM columns of a
+// slot block by block, summing one block while the next is in flight, and releases the
+// slot once its last block has landed, so the MMAs of the next slot use overlap the rest of
+// the arithmetic.  Each CTA owns one KV head and claims its key tiles from a counter shared by the
 // head's CTAs.  Every wait on an mbarrier is bounded in time:
 // on expiry the kernel records SGDKV_ERR_TIMEOUT, all roles leave their loops, in-flight
 // copies and MMAs are drained (again bounded) and TMEM is freed.
