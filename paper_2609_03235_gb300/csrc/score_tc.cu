@@ -6,10 +6,10 @@
 // the G*W window rows r = g*W + w of KV head h (contiguous in q_win):
 //
 //   pass 1 (score_pass1_tc): D[r][j] = Q_h K_tile^T, window rows on TMEM lanes and keys on
-//     columns (MMA N = 128 keys; row tiles in pairs per TMEM slot).  Every epilogue thread
-//     keeps an online (max m_r, sum Z_r = sum 2^(t_rj - m_r)) for its window rows over its
-//     share of the CTA's keys; the four shares of a row are merged in shared memory and
-//     one partial per CTA goes to the workspace.
+//     columns (MMA N = 128 keys; one 128-column TMEM slot per epilogue warpgroup, each
+//     warpgroup owning one row tile).  Every epilogue thread keeps an online (max m_r, sum
+//     Z_r = sum 2^(t_rj - m_r)) for its window row over all keys of the key tiles it
+//     receives; one partial per row per CTA goes to the workspace.
 //   pass 2 (score_pass2_tc): merges the partials into lse_r = m_r + log2 Z_r, then
 //     D[j][r] = K_tile Q_h^T (keys on TMEM lanes, rows on columns, Q_h in shared memory);
 //     every epilogue thread sums 2^(t_rj - lse_r) for its key over a quarter of the window
@@ -23,7 +23,8 @@
 // quarters that carry less epilogue work.  An epilogue warp loads its TMEM columns of a
 // slot block by block, summing one block while the next is in flight, and releases the
 // slot once its last block has landed, so the MMAs of the next slot use overlap the rest of
-// the arithmetic.  Each CTA owns one KV head and claims its key tiles from a counter shared by the
+// the arithmetic.  Pass 1 has four slots of 128 columns (one per epilogue warpgroup), pass 2
+// two of 256 shared by all sixteen epilogue warps.  Each CTA owns one KV head and claims its key tiles from a counter shared by the
 // head's CTAs.  Every wait on an mbarrier is bounded in time:
 // on expiry the kernel records SGDKV_ERR_TIMEOUT, all roles leave their loops, in-flight
 // copies and MMAs are drained (again bounded) and TMEM is freed.
@@ -50,8 +51,10 @@ constexpr uint32_t kTmemCols = 512;
 constexpr int kStageBytes = kTileKeys * 256;      // 32 KB: two 128-byte column halves
 constexpr int kHalfBytes = kTileKeys * 128;       // 16 KB
 constexpr int kMaxStages = 8;
-constexpr int kNumBars = 2 * kMaxStages + 7;      // kfull kempty tfull[2] tempty[2] qfull drain never
-constexpr int kCtlBytes = 256;                    // barriers, TMEM address, abort flag, tile ids
+constexpr int kTmemSlots = 4;                     // TMEM slots (pass 1: 4 x 128 columns, pass 2: 2 x 256)
+constexpr int kNumBars = 2 * kMaxStages + 2 * kTmemSlots + 3;   // kfull kempty tfull tempty qfull drain never
+constexpr int kCtlBytes = 512;                    // barriers, TMEM address, abort flag, tile ids
+static_assert(kNumBars * 8 + 8 + (kMaxStages + kTmemSlots) * 4 <= kCtlBytes, "control block");
 constexpr int kSmemLimit = 232448;                // opt-in dynamic shared memory per CTA
 constexpr int kQBoxRows = 32;                     // TMA box height for Q rows (pass 2)
 constexpr uint32_t kFlagStallMma = 1u;            // test hook: MMA thread waits on `never`
@@ -315,7 +318,7 @@ struct Smem {
   uint32_t* tmem_slot;
   int* abort_flag;
   volatile int* stile; // [kMaxStages] key tile held by each K stage (-1: no more tiles)
-  volatile int* utile; // [2] key tile whose products fill each TMEM slot (-1: done)
+  volatile int* utile; // [kTmemSlots] key tile whose products fill each TMEM slot (-1: done)
   float* tail;         // pass 2: -lse2[kMaxRows] (16-byte aligned)
   int qrows;
 };
@@ -337,13 +340,15 @@ __device__ __forceinline__ Smem carve(uint8_t* base, int qrows, int nstages) {
 __device__ __forceinline__ uint32_t bar_kfull(const Smem& s, int i) { return smem_u32(s.bars + i); }
 __device__ __forceinline__ uint32_t bar_kempty(const Smem& s, int i) { return smem_u32(s.bars + kMaxStages + i); }
 __device__ __forceinline__ uint32_t bar_tfull(const Smem& s, int i) { return smem_u32(s.bars + 2 * kMaxStages + i); }
-__device__ __forceinline__ uint32_t bar_tempty(const Smem& s, int i) { return smem_u32(s.bars + 2 * kMaxStages + 2 + i); }
-__device__ __forceinline__ uint32_t bar_qfull(const Smem& s) { return smem_u32(s.bars + 2 * kMaxStages + 4); }
-__device__ __forceinline__ uint32_t bar_drain(const Smem& s) { return smem_u32(s.bars + 2 * kMaxStages + 5); }
-__device__ __forceinline__ uint32_t bar_never(const Smem& s) { return smem_u32(s.bars + 2 * kMaxStages + 6); }
+__device__ __forceinline__ uint32_t bar_tempty(const Smem& s, int i) { return smem_u32(s.bars + 2 * kMaxStages + kTmemSlots + i); }
+__device__ __forceinline__ uint32_t bar_qfull(const Smem& s) { return smem_u32(s.bars + 2 * kMaxStages + 2 * kTmemSlots); }
+__device__ __forceinline__ uint32_t bar_drain(const Smem& s) { return smem_u32(s.bars + 2 * kMaxStages + 2 * kTmemSlots + 1); }
+__device__ __forceinline__ uint32_t bar_never(const Smem& s) { return smem_u32(s.bars + 2 * kMaxStages + 2 * kTmemSlots + 2); }
 
 // Barrier init, TMEM allocation; returns the TMEM base address (all threads).
-__device__ __forceinline__ uint32_t setup(const Smem& s, int nstages, uint32_t qfull_count) {
+// nslots TMEM slots whose tempty barriers expect `consumers` warp arrivals each.
+__device__ __forceinline__ uint32_t setup(const Smem& s, int nstages, uint32_t qfull_count,
+                                          int nslots, uint32_t consumers) {
   const int warp = threadIdx.x >> 5;
   if (threadIdx.x == 0) {
     for (int i = 0; i < nstages; ++i) {
@@ -351,9 +356,9 @@ __device__ __forceinline__ uint32_t setup(const Smem& s, int nstages, uint32_t q
       mbar_init(bar_kempty(s, i), 1);
     }
     // tfull: one plain arrive of the MMA thread (publishing utile) + its MMA commit
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < nslots; ++i) {
       mbar_init(bar_tfull(s, i), 2);
-      mbar_init(bar_tempty(s, i), kEpiWarps);
+      mbar_init(bar_tempty(s, i), consumers);
     }
     mbar_init(bar_qfull(s), qfull_count);
     mbar_init(bar_drain(s), 1);
@@ -517,15 +522,20 @@ __device__ __forceinline__ void online_fold(uint32_t (&v)[N], int kb, bool edge,
   Z += zc;
 }
 
-// NRT: row tiles of 128 window rows (1..4), taken in groups of two.  Q_h (padded to
-// NRT x 128 rows) sits in shared memory as the MMA's A operand, K tiles are B.  Each
-// (128-key tile, row group) fills one TMEM slot of 256 columns: D[rows][keys] for the
-// group's row tiles side by side, MMA M = 128 rows, N = 128 keys.  The two slots alternate.
+// NRT: row tiles of 128 window rows (1..4).  Q_h (padded to NRT x 128 rows) sits in shared
+// memory as the MMA's A operand, K tiles are B.  TMEM holds four slots of 128 columns, one per
+// epilogue warpgroup (the four warps wi of the lane quarters): warpgroup w takes row tile
+// w % NRT of the key tiles n with n % NB == w / NRT (NB = 4 / NRT warpgroups share a row
+// tile, taking alternate key tiles; for NRT = 3 warpgroup 3 has no work).  Per key tile the
+// MMA fills the slots of that tile's warpgroups (M = 128 rows, N = 128 keys), and each warp
+// folds all 128 keys into the (max, sum) of its 32 rows: one slot wait and one release per
+// key tile, one running (m, Z) per thread.
 template <int NRT>
 __global__ void __maxnreg__(kMaxRegs)
 score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                TcParams p, Ws ws) {
-  constexpr int NG = (NRT + 1) / 2;            // row groups (slot uses per key tile)
+  constexpr int NB = 4 / NRT;                  // key-tile phases (warpgroups per row tile)
+  constexpr int NWG = NRT * NB;                // warpgroups with work
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   if (smem_u32(smem_raw) & 1023u) {
     if (threadIdx.x == 0) record_error(ws.status, SGDKV_ERR_INTERNAL);
@@ -535,7 +545,7 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   const int h = blockIdx.x / p.cph, ci = blockIdx.x % p.cph;
   uint32_t* counter = ws.sched + h;
   const Smem s = carve(smem_raw, NRT * 128, p.nstages);
-  const uint32_t tmem = setup(s, p.nstages, 1);
+  const uint32_t tmem = setup(s, p.nstages, 1, kTmemSlots, 4);
   volatile int* ab = s.abort_flag;
 
   if (warp == kProducerWarp) {
@@ -545,110 +555,95 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     const uint32_t idesc = idesc_bf16(128, kTileKeys);
     bool ok = mma_start(s, p, ws.status);
     const uint32_t q_lo = desc_lo(smem_u32(s.q)), qhalf = uint32_t(s.qrows * 128);
+    int fills[kTmemSlots] = {0, 0, 0, 0};        // uses of each slot so far
     for (int n = 0; ok; ++n) {
       const int st = n % p.nstages;
       if (!(ok = wwait(bar_kfull(s, st), (n / p.nstages) & 1, ab, p.wait_ns, ws.status))) break;
       tc_fence_after();
       const int tile = s.stile[st];
       const uint32_t k_lo = desc_lo(smem_u32(s.k + st * kStageBytes));
+      const int ph = n % NB;
 #pragma unroll
-      for (int g = 0; g < NG; ++g) {
-        const int u = n * NG + g, slot = u & 1;
-        if (!(ok = wwait(bar_tempty(s, slot), ((u >> 1) & 1) ^ 1, ab, p.wait_ns, ws.status)))
-          break;
+      for (int w = 0; w < NWG; ++w) {
+        if (tile >= 0 && w / NRT != ph) continue;   // the end (tile -1) goes to every slot
+        if (!(ok = wwait(bar_tempty(s, w), (fills[w] & 1) ^ 1, ab, p.wait_ns, ws.status))) break;
         tc_fence_after();
-        publish_slot(s, slot, tile, leader);
-        if (tile < 0) break;
-#pragma unroll
-        for (int i = 0; i < 2; ++i)
-          if (2 * g + i < NRT)
-            umma_k128(tmem + uint32_t(slot * 256 + i * kTileKeys),
-                      q_lo + uint32_t(2 * g + i) * (kHalfBytes >> 4), qhalf >> 4, k_lo,
-                      kHalfBytes >> 4, idesc, leader);
-        umma_commit(bar_tfull(s, slot), leader);
+        publish_slot(s, w, tile, leader);
+        ++fills[w];
+        if (tile < 0) continue;
+        umma_k128(tmem + uint32_t(w * kTileKeys), q_lo + uint32_t(w % NRT) * (kHalfBytes >> 4),
+                  qhalf >> 4, k_lo, kHalfBytes >> 4, idesc, leader);
+        umma_commit(bar_tfull(s, w), leader);
       }
-      if (tile < 0) break;
-      if (ok) umma_commit(bar_kempty(s, st), leader);
+      if (tile < 0 || !ok) break;
+      umma_commit(bar_kempty(s, st), leader);
     }
     if (!ok) mma_drain(s, leader, ws.status);
   } else if (warp >= kFirstEpiWarp) {
-    // Epilogue: the 4 warps of a TMEM lane quarter q share its 32 rows of every row tile
-    // and split each slot's 128 keys into 4 blocks of 32.
     const int q = warp & 3, wi = (warp - kFirstEpiWarp) >> 2;
+    const int rt = wi % NRT, ph = wi / NRT;
+    const int r = rt * 128 + 32 * q + lane;              // this thread's window row
+    const bool valid = wi < NWG && rt * 128 + 32 * q < p.GW;   // warp-uniform
     // keys above a row's limit are masked; lim_base: the lowest limit of any row
     const int lim_base = p.causal ? int(p.L - p.W) : int(p.L - 1);   // Hkv * L < 2^31
-    float m[NRT], Z[NRT];
-    int lim[NRT];
-    bool valid[NRT];
-#pragma unroll
-    for (int rt = 0; rt < NRT; ++rt) {
-      m[rt] = -INFINITY;
-      Z[rt] = 0.f;
-      valid[rt] = rt * 128 + 32 * q < p.GW;                  // warp-uniform
-      lim[rt] = p.causal ? lim_base + (rt * 128 + 32 * q + lane) % p.W : lim_base;
-    }
-    bool ok = true;
-    for (int n = 0; ok; ++n) {
-#pragma unroll
-      for (int g = 0; g < NG; ++g) {
-        const int u = n * NG + g, slot = u & 1;
-        if (!(ok = bwait(bar_tfull(s, slot), (u >> 1) & 1, ab, p.wait_ns, ws.status))) break;
+    const int lim = p.causal ? lim_base + r % p.W : lim_base;
+    float m = -INFINITY, Z = 0.f;
+    if (wi < NWG) {
+      const uint32_t tf = bar_tfull(s, wi), te = bar_tempty(s, wi);
+      const uint32_t tb = tmem + (uint32_t(32 * q) << 16) + uint32_t(wi * kTileKeys);
+      for (int c = 0;; ++c) {
+        if (!bwait(tf, c & 1, ab, p.wait_ns, ws.status)) break;
         tc_fence_after();
-        const int tile = s.utile[slot];
-        if (tile < 0) {
-          ok = false;                              // no more tiles: leave both loops
-          break;
-        }
-        const int kb = tile * kTileKeys + wi * 32;
-        const bool edge = kb + 31 > lim_base;
-        uint32_t v[2][32];
-        const uint32_t tb = tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256 + wi * 32);
-        // The second row tile's load is in flight while the first is folded; the slot is
-        // released once both have landed.
-        const int rt0 = 2 * g, rt1 = 2 * g + 1;
-        const bool h0 = rt0 < NRT && valid[rt0], h1 = rt1 < NRT && valid[rt1];
-        if (h0) {
-          tmem_ld32(tb, v[0]);
-          tmem_wait_ld(v[0]);
-        }
-        if (h1) tmem_ld32(tb + uint32_t(kTileKeys), v[1]);
+        const int tile = s.utile[wi];
+        if (tile < 0) break;                             // no more tiles
         auto release = [&] {
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive(bar_tempty(s, slot));
+          if (lane == 0) mbar_arrive(te);
         };
-        if (!h1) release();
-        if (h0) online_fold<32>(v[0], kb, edge, lim[rt0], p.scale2, m[rt0], Z[rt0]);
-        if (h1) {
-          tmem_wait_ld(v[1]);
+        if (!valid) {
           release();
-          online_fold<32>(v[1], kb, edge, lim[rt1], p.scale2, m[rt1], Z[rt1]);
+          continue;
+        }
+        // 4 blocks of 32 keys: block b + 1 in flight while block b is folded; the slot is
+        // released once the last block has landed.
+        const int kb = tile * kTileKeys;
+        uint32_t v[2][32];
+        tmem_ld32(tb, v[0]);
+        tmem_wait_ld(v[0]);
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+          if (b < 3) tmem_ld32(tb + uint32_t(32 * (b + 1)), v[(b + 1) & 1]);
+          else release();
+          online_fold<32>(v[b & 1], kb + 32 * b, kb + 32 * b + 31 > lim_base, lim, p.scale2, m,
+                          Z);
+          if (b < 3) tmem_wait_ld(v[(b + 1) & 1]);
         }
       }
     }
-    // Merge the 4 key shares of every row in shared memory (the K ring is idle by now: all
-    // tiles were consumed) and write one partial per row per CTA.
-    float2* red = reinterpret_cast<float2*>(s.k);           // [4][kMaxRows]
+    // The NB warpgroups of a row tile merge their (m, Z) in shared memory, in the K ring:
+    // once every epilogue warp has seen the end of its slot, the last MMA of every slot has
+    // completed and the ring is idle.  One partial per row per CTA.
+    float2* red = reinterpret_cast<float2*>(s.k);           // [NB][kMaxRows]
+    if (NB > 1) {
+      asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+      if (valid && !*ab) red[ph * kMaxRows + r] = make_float2(m, Z);
+      asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+    }
+    if (valid && ph == 0 && !*ab) {
+      float M = m, S = Z;
+      if (NB > 1) {
+        M = -INFINITY;
 #pragma unroll
-    for (int rt = 0; rt < NRT; ++rt)
-      if (valid[rt]) red[wi * kMaxRows + rt * 128 + 32 * q + lane] = make_float2(m[rt], Z[rt]);
-    asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
-    if (wi == 0 && !*ab) {
+        for (int i = 0; i < NB; ++i) M = fmaxf(M, red[i * kMaxRows + r].x);
+        S = 0.f;
 #pragma unroll
-      for (int rt = 0; rt < NRT; ++rt) {
-        if (!valid[rt]) continue;
-        const int r = rt * 128 + 32 * q + lane;
-        float M = -INFINITY;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) M = fmaxf(M, red[i * kMaxRows + r].x);
-        float S = 0.f;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
+        for (int i = 0; i < NB; ++i) {
           const float2 e = red[i * kMaxRows + r];
           if (e.x != -INFINITY) S += e.y * ex2(e.x - M);
         }
-        ws.partial[(int64_t(h) * kMaxScoreParts + ci) * kMaxRows + r] = make_float2(M, S);
       }
+      ws.partial[(int64_t(h) * kMaxScoreParts + ci) * kMaxRows + r] = make_float2(M, S);
     }
   }
   teardown(tmem);
@@ -706,7 +701,7 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   uint32_t* counter = ws.sched + 2 * SGDKV_MAX_KV_HEADS + h;
   const Smem s = carve(smem_raw, p.GW, p.nstages);
   float* lse2 = s.tail;                          // [kMaxRows], negated
-  const uint32_t tmem = setup(s, p.nstages, 1);
+  const uint32_t tmem = setup(s, p.nstages, 1, 2, kEpiWarps);
   volatile int* ab = s.abort_flag;
   const int nch = p.GW > 256 ? 2 : 1;            // N chunks of the window rows per tile
   const int nn = p.GW / nch;                     // MMA N
