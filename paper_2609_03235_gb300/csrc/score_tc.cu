@@ -899,25 +899,62 @@ maxpool_sum_kernel(const float* __restrict__ raw, float* __restrict__ out, int64
   const int h = int(blockIdx.x / tiles);
   const int64_t base = (blockIdx.x % tiles) * kPoolTile;
   const float* r0 = raw + int64_t(h) * L;
+  auto comb = [&](float a, float b, float c, float d) {
+    return combine_max ? fmaxf(fmaxf(a, b), fmaxf(c, d)) : (a + b) + (c + d);
+  };
+  auto at = [&](int64_t j) {                       // plane combination at position j
+    return comb(__ldcg(r0 + j), __ldcg(r0 + plane + j), __ldcg(r0 + 2 * plane + j),
+                __ldcg(r0 + 3 * plane + j));
+  };
+  // sum[i] holds position base - radius + i (-inf outside the row)
   const int span = kPoolTile + 2 * radius;
-  for (int i = threadIdx.x; i < span; i += kPoolThreads) {
-    const int64_t j = base - radius + i;
-    float v = -INFINITY;
-    if (j >= 0 && j < L) {
-      const float a = __ldcg(r0 + j), b = __ldcg(r0 + plane + j);
-      const float c = __ldcg(r0 + 2 * plane + j), d = __ldcg(r0 + 3 * plane + j);
-      v = combine_max ? fmaxf(fmaxf(a, b), fmaxf(c, d)) : (a + b) + (c + d);
+  // whole tile, rows a multiple of 4 positions long and 16-byte aligned buffers: one 16-byte
+  // load per plane per thread (and one 16-byte store), the halo by scalar loads
+  const bool vec = (L & 3) == 0 && base + kPoolTile <= L &&
+                   ((reinterpret_cast<uintptr_t>(raw) | reinterpret_cast<uintptr_t>(out)) & 15) == 0;
+  if (vec) {
+    static_assert(kPoolTile == 4 * kPoolThreads, "four positions per thread");
+    const int t = threadIdx.x;
+    const int64_t j = base + 4 * t;
+    const float4 a = __ldcg(reinterpret_cast<const float4*>(r0 + j));
+    const float4 b = __ldcg(reinterpret_cast<const float4*>(r0 + plane + j));
+    const float4 c = __ldcg(reinterpret_cast<const float4*>(r0 + 2 * plane + j));
+    const float4 d = __ldcg(reinterpret_cast<const float4*>(r0 + 3 * plane + j));
+    float* sp = sum + radius + 4 * t;
+    sp[0] = comb(a.x, b.x, c.x, d.x);
+    sp[1] = comb(a.y, b.y, c.y, d.y);
+    sp[2] = comb(a.z, b.z, c.z, d.z);
+    sp[3] = comb(a.w, b.w, c.w, d.w);
+    if (t < 2 * radius) {
+      const int i = t < radius ? t : kPoolTile + t;
+      const int64_t jh = base - radius + i;
+      sum[i] = jh >= 0 && jh < L ? at(jh) : -INFINITY;
     }
-    sum[i] = v;
+  } else {
+    for (int i = threadIdx.x; i < span; i += kPoolThreads) {
+      const int64_t jh = base - radius + i;
+      sum[i] = jh >= 0 && jh < L ? at(jh) : -INFINITY;
+    }
   }
   __syncthreads();
   float* o = out + int64_t(h) * L;
-  for (int i = threadIdx.x; i < kPoolTile; i += kPoolThreads) {
-    const int64_t j = base + i;
-    if (j >= L) break;
-    float m = sum[i + radius];
-    for (int k = 0; k < 2 * radius + 1; ++k) m = fmaxf(m, sum[i + k]);
-    o[j] = m;
+  if (vec) {
+    const int i0 = 4 * threadIdx.x;
+    float m[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) m[e] = sum[i0 + e + radius];
+    for (int k = 0; k < 2 * radius + 1; ++k)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) m[e] = fmaxf(m[e], sum[i0 + e + k]);
+    *reinterpret_cast<float4*>(o + base + i0) = make_float4(m[0], m[1], m[2], m[3]);
+  } else {
+    for (int i = threadIdx.x; i < kPoolTile; i += kPoolThreads) {
+      const int64_t j = base + i;
+      if (j >= L) break;
+      float m = sum[i + radius];
+      for (int k = 0; k < 2 * radius + 1; ++k) m = fmaxf(m, sum[i + k]);
+      o[j] = m;
+    }
   }
 }
 

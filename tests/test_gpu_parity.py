@@ -65,6 +65,24 @@ def test_score_parity(dev, Hq, Hkv, L, W, pool):
     assert ok.all(), f"{(~ok).sum()} of {ok.size} off; worst {np.max(np.abs(got - exp))}"
 
 
+def test_score_output_not_16_byte_aligned_is_refused(dev):
+    """scores_out 4 bytes past a 16-byte boundary: INVALID_ARG, nothing launched, the buffer
+    untouched (the pooled scores are written with 16-byte stores)."""
+    Hq, Hkv, L, W = 28, 4, 4096, 64
+    wl = synth.tiny_workload(Hq=Hq, Hkv=Hkv, d=128, L=L, W=W, n_salient=8)
+    inp = synth.tiny_inputs(wl, tag=77)
+    q, K, _ = _upload(inp, dev)
+    ws = sg.make_workspace(Hq, Hkv, L, W, dev)
+    buf = torch.full((Hkv * L + 1,), float("nan"), dtype=torch.float32, device=dev)
+    out = buf[1:].view(Hkv, L)
+    assert out.data_ptr() % 16 == 4
+    with pytest.raises(sg.SgdkvError) as e:
+        sg.sgdkv_score(q, K, W, 7, out, ws)
+    assert e.value.status == sg.ERR_INVALID_ARG
+    torch.cuda.synchronize()
+    assert torch.isnan(buf).all()
+
+
 PROXY_SHAPES = [
     # Hq, Hkv, L, W    (W external query rows per query head; every row sees all L keys)
     (14, 2, 1000, 32),
