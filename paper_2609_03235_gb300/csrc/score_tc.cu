@@ -789,6 +789,10 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     const int gpc = nn / 16;                     // 16-column blocks per chunk (<= 16)
     float* raw_out = ws.raw + int64_t(wi) * p.Hkv * p.L + int64_t(h) * p.L;
     const int lim_base = p.causal ? int(p.L - p.W) : int(p.L - 1);   // lowest row limit
+    // this warp's first block and block count in chunks 0 and 1 (loop invariants)
+    const int li0_0 = wi, li0_1 = (((wi - gpc) % 4) + 4) % 4;
+    const int ng_0 = li0_0 < gpc ? (gpc - li0_0 + 3) / 4 : 0;
+    const int ng_1 = li0_1 < gpc ? (gpc - li0_1 + 3) / 4 : 0;
     bool ok = true;
     for (int n = 0; ok; ++n) {
       int j = 0;
@@ -811,8 +815,8 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
           for (int b = 0; b < gpc && ng < 4; ++b)
             if (((c * nn + 16 * b) / p.W) % 4 == wi) blk[ng++] = b;
         } else {
-          li0 = (((wi - c * gpc) % 4) + 4) % 4;   // first block of this warp in chunk c
-          ng = li0 < gpc ? (gpc - li0 + 3) / 4 : 0;
+          li0 = c ? li0_1 : li0_0;                // first block of this warp in chunk c
+          ng = c ? ng_1 : ng_0;
         }
         const uint32_t tb = tmem + (uint32_t(32 * q) << 16) + uint32_t(slot * 256);
         if (!PERG && !masked && ng > 0) {
