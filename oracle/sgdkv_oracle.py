@@ -12,7 +12,11 @@ Steps and the passages they follow (SGD-KV, "Summarization Guided KV Cache Compr
   sink + window floor, proportional share of the middle, Eq. 2) and Appendix A.1,
   Algorithm 1 (cap at the middle length, collect the excess, hand it to the remaining
   heads in descending score order).  Integer rounding is not stated by the paper; the
-  reading used is largest remainder (ties: higher score, then lower head index).
+  reading used is largest remainder (ties: higher score, then lower head index).  Modes
+  after the appendix's ablation (Table 3): "thr" (scores below the mean zeroed first) and
+  "Reverse" (every head's middle share inverted).
+* ``mix_head_scores``: the "SGD-KV + HeadKV" row of the same ablation: the normalised
+  summarization scores and the normalised HeadKV retrieval-reasoning scores, averaged.
 * ``window_scores``: Section 3.3 and Section 5 (token selection from the cumulative
   attention of a final observation window, SnapKV-style): softmax over the causal keys of
   each window query, summed over the window and over the query heads of the KV head's
@@ -39,7 +43,7 @@ import math
 
 import numpy as np
 
-GREEDY, PROPORTIONAL, THRESHOLD = 0, 1, 2
+GREEDY, PROPORTIONAL, THRESHOLD, REVERSE = 0, 1, 2, 3
 AGG_SUM, AGG_IPT_MAX, AGG_IPT_MEAN, AGG_IPT_ONLY = 0, 1, 2, 3
 
 
@@ -136,7 +140,10 @@ def allocate_budgets(head_scores, context_len: int, total_budget: int, floor: in
     (R = P / (N M)).  Appendix A.1 (Algorithm 1) then caps each middle share at M and
     redistributes the excess.  mode 0: greedy redistribution (default reading);
     mode 1: proportional water filling; mode 2: "thr" variant of the appendix (scores below
-    the mean set to zero first), then greedy.
+    the mean set to zero first), then greedy; mode 3: "Reverse" row of the appendix's
+    ablation (Table 3): the greedy allocation of T with every head's middle share m_h
+    inverted to M - m_h (a head given 10 % of its middle keeps 90 %), floors kept, so the
+    budgets sum to N (C + f) - T.
     """
     n = len(head_scores)
     C, T, f = int(context_len), int(total_budget), int(floor)
@@ -155,14 +162,27 @@ def allocate_budgets(head_scores, context_len: int, total_budget: int, floor: in
     cap = C - f
     pool = T - n * f
     x = [S[h] * pool for h in range(n)]
-    if mode in (GREEDY, THRESHOLD):
+    if mode in (GREEDY, THRESHOLD, REVERSE):
         xt = _greedy_redistribute(S, x, float(cap))
     elif mode == PROPORTIONAL:
         xt = _proportional_waterfill(S, float(pool), float(cap))
     else:
         raise ValueError("unknown mode")
     m = _largest_remainder(S, xt, pool, cap)
+    if mode == REVERSE:
+        m = [cap - v for v in m]
     return np.asarray([f + v for v in m], dtype=np.int64)
+
+
+def mix_head_scores(a, b) -> np.ndarray:
+    """Scores of the "SGD-KV + HeadKV" row of the appendix's ablation (Table 3): the two
+    per-head score sets (summarization scores and the retrieval-reasoning scores of HeadKV)
+    are each normalised to sum one over all heads and averaged: (a_h/sum a + b_h/sum b) / 2.
+    float32 in, float32 out (the average formed in float64, rounded once)."""
+    A, B = normalise(a), normalise(b)
+    if len(A) != len(B):
+        raise ValueError("score sets differ in length")
+    return np.asarray([(A[h] + B[h]) / 2.0 for h in range(len(A))], dtype=np.float32)
 
 
 # ----------------------------------------------------------------------------------------

@@ -152,3 +152,58 @@ def test_rejects_infeasible():
         O.allocate_budgets(s, 100, 4 * 10 - 1, 10)
     with pytest.raises(ValueError):
         O.allocate_budgets(s, 100, 4 * 100 + 1, 10)
+
+
+def test_reverse_at_a_quarter_is_three_times_the_cache():
+    """Appendix ablation (Table 3): SGD-KV (Reverse) is compared 'even with 3x KV cache':
+    with no floor, reversing an allocation of 25 % of every head's keys keeps 75 %."""
+    rng = np.random.default_rng(5)
+    n, C = 112, 4096
+    s = rng.gamma(0.7, size=n).astype(np.float32)
+    T = n * C // 4
+    fwd = O.allocate_budgets(s, C, T, 0, O.GREEDY)
+    rev = O.allocate_budgets(s, C, T, 0, O.REVERSE)
+    assert int(rev.sum()) == 3 * T
+    assert np.all(rev == C - fwd)
+    # the head with the largest forward budget has the smallest reverse one
+    assert int(np.argmax(fwd)) == int(np.argmin(rev))
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_reverse_bounds_and_order(seed):
+    """Reversed budgets stay within [f, C] and reverse the forward order of the heads."""
+    rng = np.random.default_rng(100 + seed)
+    n, C, f = 40, 2000, 128
+    s = rng.gamma(0.5, size=n).astype(np.float32)
+    T = int(rng.integers(n * f, n * C))
+    fwd = O.allocate_budgets(s, C, T, f, O.GREEDY)
+    rev = O.allocate_budgets(s, C, T, f, O.REVERSE)
+    assert np.all(rev >= f) and np.all(rev <= C)
+    assert int(rev.sum()) == n * (C + f) - T
+    for a in range(n):
+        for b in range(n):
+            if fwd[a] > fwd[b]:
+                assert rev[a] < rev[b]
+
+
+def test_mix_head_scores_closed_forms():
+    """SGD-KV + HeadKV (appendix ablation): the average of the two normalised score sets.
+    Mirror-image sets mix to uniform; an all-zero set counts as uniform; a set mixed with
+    itself is its own normalisation; the mix sums to one."""
+    assert O.mix_head_scores([1, 3], [3, 1]).tolist() == [0.5, 0.5]
+    assert O.mix_head_scores([0, 0], [1, 3]).tolist() == [0.375, 0.625]
+    rng = np.random.default_rng(9)
+    a = rng.gamma(0.8, size=50).astype(np.float32)
+    b = rng.gamma(0.8, size=50).astype(np.float32)
+    np.testing.assert_array_equal(O.mix_head_scores(a, a), np.float32(O.normalise(a)))
+    assert abs(float(np.sum(O.mix_head_scores(a, b), dtype=np.float64)) - 1.0) < 1e-5
+    # a head that both sets rank first also ranks first in the mix
+    a[7] = b[7] = 100.0
+    assert int(np.argmax(O.mix_head_scores(a, b))) == 7
+
+
+def test_mix_head_scores_rejects_bad_input():
+    with pytest.raises(ValueError):
+        O.mix_head_scores([1, -1], [1, 1])
+    with pytest.raises(ValueError):
+        O.mix_head_scores([1, 2], [1, 2, 3])
