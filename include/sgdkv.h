@@ -66,6 +66,7 @@ typedef enum {
 #define SGDKV_ALLOC_GREEDY 0       /* Algorithm 1, excess to top-scoring heads in turn     */
 #define SGDKV_ALLOC_PROPORTIONAL 1 /* water level: min(cap, lambda * S_h)                  */
 #define SGDKV_ALLOC_THRESHOLD 2    /* appendix "thr": scores below the mean zeroed, greedy */
+#define SGDKV_ALLOC_REVERSE 3      /* appendix "Reverse": greedy, every middle share inverted */
 
 /* Static description of a status code. Never NULL. */
 SGDKV_API const char* sgdkv_status_string(int status);
@@ -90,6 +91,9 @@ SGDKV_API int sgdkv_version(void);
  * The middle pool P = T - n_heads*f is shared in proportion to S_h = s_h / sum(s)
  * (Eq. 2), shares above M are capped and their excess redistributed (Algorithm 1), and
  * the real shares are rounded by largest remainder (ties: higher S_h, then lower index).
+ * SGDKV_ALLOC_REVERSE (the "SGD-KV (Reverse)" row of the appendix's ablation, Table 3):
+ * the greedy allocation of T, then every head's middle share m_h = b_h - f becomes M - m_h
+ * (a head given 10 % keeps 90 %), so for this mode sum b_h == n*(C + f) - T instead.
  * All arithmetic is IEEE double in a fixed order, so results are bit-reproducible.
  * Errors: INVALID_ARG (null, n_heads <= 0, f outside [0, C], bad mode, negative/NaN/Inf
  * score), INFEASIBLE_BUDGET (T outside [n*f, n*C]).  budgets_out untouched on error.
@@ -97,6 +101,19 @@ SGDKV_API int sgdkv_version(void);
 SGDKV_API sgdkv_status sgdkv_allocate_budgets(const float* head_scores, int32_t n_heads,
                                     int64_t context_len, int64_t total_budget, int64_t floor,
                                     int32_t mode, int64_t* budgets_out);
+
+/*
+ * Head scores of the "SGD-KV + HeadKV" row of the appendix's ablation (Table 3): two score
+ * sets over the same heads (summarization scores and HeadKV's retrieval-reasoning scores),
+ * each normalised to sum one (an all-zero set counts as uniform), then averaged:
+ *   scores_out[h] = (a[h] / sum(a) + b[h] / sum(b)) / 2
+ * with the sums taken in ascending head order in IEEE double and the result rounded once
+ * to float.  The output is a head_scores input of sgdkv_allocate_budgets.  Host only.
+ * a, b, scores_out  [n_heads] host floats (scores_out may alias a or b).
+ * Errors: INVALID_ARG (null, n_heads <= 0, negative/NaN/Inf score); scores_out untouched.
+ */
+SGDKV_API sgdkv_status sgdkv_mix_head_scores(const float* a, const float* b, int32_t n_heads,
+                                             float* scores_out);
 
 /* Workspace bytes needed by sgdkv_score / sgdkv_compact / sgdkv_compress_layer for this
  * shape (one size serves all three).  Returns 0 for shapes outside the v1 limits. */

@@ -132,7 +132,7 @@ extern "C" sgdkv_status sgdkv_allocate_budgets(const float* head_scores, int32_t
   if (!head_scores || !budgets_out || n_heads <= 0) return SGDKV_ERR_INVALID_ARG;
   if (context_len <= 0 || context_len > (int64_t(1) << 40)) return SGDKV_ERR_INVALID_ARG;
   if (floor < 0 || floor > context_len) return SGDKV_ERR_INVALID_ARG;
-  if (mode < SGDKV_ALLOC_GREEDY || mode > SGDKV_ALLOC_THRESHOLD) return SGDKV_ERR_INVALID_ARG;
+  if (mode < SGDKV_ALLOC_GREEDY || mode > SGDKV_ALLOC_REVERSE) return SGDKV_ERR_INVALID_ARG;
   const int n = n_heads;
   std::vector<double> s(n);
   for (int h = 0; h < n; ++h) {
@@ -161,6 +161,24 @@ extern "C" sgdkv_status sgdkv_allocate_budgets(const float* head_scores, int32_t
                                : greedy_redistribute(S, x, double(cap));
   std::vector<int64_t> m;
   if (!largest_remainder(S, xt, pool, cap, m)) return SGDKV_ERR_INFEASIBLE_BUDGET;
-  for (int h = 0; h < n; ++h) budgets_out[h] = f + m[h];
+  for (int h = 0; h < n; ++h)
+    budgets_out[h] = f + (mode == SGDKV_ALLOC_REVERSE ? cap - m[h] : m[h]);
+  return SGDKV_OK;
+}
+
+// SGD-KV + HeadKV scores: the mean of the two normalised score sets.
+extern "C" sgdkv_status sgdkv_mix_head_scores(const float* a, const float* b, int32_t n_heads,
+                                              float* scores_out) {
+  if (!a || !b || !scores_out || n_heads <= 0) return SGDKV_ERR_INVALID_ARG;
+  const int n = n_heads;
+  std::vector<double> sa(n), sb(n);
+  for (int h = 0; h < n; ++h) {
+    if (!std::isfinite(a[h]) || a[h] < 0.0f || !std::isfinite(b[h]) || b[h] < 0.0f)
+      return SGDKV_ERR_INVALID_ARG;
+    sa[h] = double(a[h]);
+    sb[h] = double(b[h]);
+  }
+  const std::vector<double> A = normalise(sa), B = normalise(sb);
+  for (int h = 0; h < n; ++h) scores_out[h] = float((A[h] + B[h]) / 2.0);
   return SGDKV_OK;
 }

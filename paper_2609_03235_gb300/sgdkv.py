@@ -16,12 +16,13 @@ LIB_PATH = os.path.join(_HERE, "lib", "libsgdkv.so")
 
 OK, ERR_INVALID_ARG, ERR_INFEASIBLE_BUDGET, ERR_WORKSPACE, ERR_CUDA, ERR_TIMEOUT, \
     ERR_UNSUPPORTED, ERR_INTERNAL = range(8)
-ALLOC_GREEDY, ALLOC_PROPORTIONAL, ALLOC_THRESHOLD = 0, 1, 2
+ALLOC_GREEDY, ALLOC_PROPORTIONAL, ALLOC_THRESHOLD, ALLOC_REVERSE = 0, 1, 2, 3
 EXPORTED = ("sgdkv_status_string", "sgdkv_version", "sgdkv_allocate_budgets",
             "sgdkv_workspace_bytes", "sgdkv_score", "sgdkv_compact", "sgdkv_compress_layer",
             "sgdkv_last_error", "sgdkv_launch_count", "sgdkv_debug_set_score_hooks",
             "sgdkv_last_cuda_error_string", "sgdkv_score_static",
-            "sgdkv_debug_enable_kernel_timing", "sgdkv_debug_kernel_timing", "sgdkv_score_ex")
+            "sgdkv_debug_enable_kernel_timing", "sgdkv_debug_kernel_timing", "sgdkv_score_ex",
+            "sgdkv_mix_head_scores")
 
 
 class LibraryMissing(RuntimeError):
@@ -54,6 +55,8 @@ def lib():
         L.sgdkv_version.restype = ctypes.c_int
         L.sgdkv_allocate_budgets.restype = ctypes.c_int
         L.sgdkv_allocate_budgets.argtypes = [_P, _I32, _I64, _I64, _I64, _I32, _P]
+        L.sgdkv_mix_head_scores.restype = ctypes.c_int
+        L.sgdkv_mix_head_scores.argtypes = [_P, _P, _I32, _P]
         L.sgdkv_workspace_bytes.restype = _SZ
         L.sgdkv_workspace_bytes.argtypes = [_I32, _I32, _I64, _I32, _I32]
         L.sgdkv_score.restype = ctypes.c_int
@@ -116,6 +119,19 @@ def sgdkv_allocate_budgets(head_scores, context_len: int, total_budget: int, flo
                                       int(total_budget), int(floor), int(mode),
                                       out.ctypes.data_as(_P))
     _check(st, "sgdkv_allocate_budgets")
+    return out
+
+
+def sgdkv_mix_head_scores(a, b) -> np.ndarray:
+    """SGD-KV + HeadKV head scores: the mean of the two normalised score sets."""
+    a = np.ascontiguousarray(a, dtype=np.float32)
+    b = np.ascontiguousarray(b, dtype=np.float32)
+    if a.size != b.size:
+        raise ValueError("score sets differ in length")
+    out = np.zeros(a.size, dtype=np.float32)
+    st = lib().sgdkv_mix_head_scores(a.ctypes.data_as(_P), b.ctypes.data_as(_P), a.size,
+                                     out.ctypes.data_as(_P))
+    _check(st, "sgdkv_mix_head_scores")
     return out
 
 

@@ -58,7 +58,8 @@ def _random_alloc_case(rng):
     return s, C, T, f
 
 
-@pytest.mark.parametrize("mode", [sg.ALLOC_GREEDY, sg.ALLOC_PROPORTIONAL, sg.ALLOC_THRESHOLD])
+@pytest.mark.parametrize("mode", [sg.ALLOC_GREEDY, sg.ALLOC_PROPORTIONAL, sg.ALLOC_THRESHOLD,
+                                  sg.ALLOC_REVERSE])
 def test_allocator_bit_exact_vs_oracle(mode):
     rng = np.random.default_rng(2024 + mode)
     for _ in range(150):
@@ -90,6 +91,31 @@ def test_allocator_errors(args, status):
     with pytest.raises(sg.SgdkvError) as e:
         sg.sgdkv_allocate_budgets(*args)
     assert e.value.status == status
+
+
+def test_mix_head_scores_bit_exact_vs_oracle():
+    rng = np.random.default_rng(77)
+    for _ in range(100):
+        n = int(rng.integers(1, 300))
+        a = (rng.gamma(0.6, size=n) * rng.choice([1e-3, 1.0, 1e3])).astype(np.float32)
+        b = (rng.gamma(0.6, size=n) * rng.choice([1e-3, 1.0, 1e3])).astype(np.float32)
+        if rng.random() < 0.1:
+            b[:] = 0.0
+        np.testing.assert_array_equal(sg.sgdkv_mix_head_scores(a, b), O.mix_head_scores(a, b))
+    # the mixed scores drive the allocator like any other head scores
+    a = rng.gamma(0.6, size=112).astype(np.float32)
+    b = rng.gamma(0.6, size=112).astype(np.float32)
+    mix = sg.sgdkv_mix_head_scores(a, b)
+    np.testing.assert_array_equal(sg.sgdkv_allocate_budgets(mix, 4096, 112 * 1024, 256),
+                                  O.allocate_budgets(O.mix_head_scores(a, b), 4096, 112 * 1024, 256))
+
+
+@pytest.mark.parametrize("a,b", [([1.0, -1.0], [1.0, 1.0]), ([1.0, 1.0], [np.inf, 1.0]),
+                                 ([np.nan, 1.0], [1.0, 1.0])])
+def test_mix_head_scores_errors(a, b):
+    with pytest.raises(sg.SgdkvError) as e:
+        sg.sgdkv_mix_head_scores(np.float32(a), np.float32(b))
+    assert e.value.status == sg.ERR_INVALID_ARG
 
 
 def test_allocator_bad_mode():
