@@ -242,8 +242,8 @@ def workload_config(wl, args, world, n_layers):
             "context_len": wl.L, "window": wl.W, "pool": wl.pool,
             "budget_frac": args.frac, "floor": wl.floor, "n_sink": n_sink,
             "n_recent": n_recent, "parallelism": f"replicas x{world}",
-            "streams": "scoring on one stream, selection + gather on a second; layer "
-                       "l's compaction overlaps layer l+1's scoring",
+            "streams": "scoring passes on one stream, max-pool + selection + gather on a "
+                       "second; layer l's pooling and compaction overlap layer l+1's scoring",
             "l2": "inputs larger than L2 (K+V of one layer = %d MiB)" %
                   (2 * wl.Hkv * wl.L * wl.d * 2 >> 20)}
 
@@ -276,20 +276,23 @@ def run_ours(args, world, rank, local):
             cu=torch.empty(wl.Hkv + 1, dtype=torch.int32, device=dev),
             ko=torch.empty((tot, wl.d), dtype=torch.bfloat16, device=dev),
             vo=torch.empty((tot, wl.d), dtype=torch.bfloat16, device=dev)))
-    # One step = the host budget allocation (a1), then the launches of every layer: scoring on
-    # the capturing stream, selection + gather on `sel_stream`; layer l's compaction waits for
-    # layer l's scores only, so it overlaps layer l+1's scoring, whose CTAs claim key tiles
-    # dynamically and absorb the SMs the compaction leaves.  The launches of a step are
+    # One step = the host budget allocation (a1), then the launches of every layer: the two
+    # scoring passes on the capturing stream, max-pool + selection + gather on `sel_stream`;
+    # layer l's pooling and compaction wait for layer l's passes only, so they overlap layer
+    # l+1's scoring, whose CTAs claim key tiles dynamically and absorb the SMs the other
+    # stream leaves.  The raw scores of layer l stay in scoring workspace l % 2 until its
+    # pool has read them (layer l + 2's scoring waits for that).  The launches of a step are
     # captured into a CUDA graph (per-kernel launch cost ~1 us instead of ~3 us on a stream)
     # and the graph is replayed; the allocation still runs on the host every step and must
     # reproduce the budgets the graph was captured with.
-    ws = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
+    ws2 = [sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev) for _ in range(2)]
     ws_sel = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
     stream = torch.cuda.current_stream(dev)
     lo_prio, hi_prio = torch.cuda.Stream.priority_range()
     sel_stream = torch.cuda.Stream(dev, priority=hi_prio)
     fork = torch.cuda.Event()
     scored = [torch.cuda.Event() for _ in range(Ls)]
+    pooled = [torch.cuda.Event() for _ in range(Ls)]
     done = torch.cuda.Event()
 
     def launches(ball, s, kinds=(), every=1, first=0):
@@ -299,9 +302,14 @@ def run_ours(args, world, rank, local):
             inp, o = layers[l], outs[l]
             b = ball[l * wl.Hkv:(l + 1) * wl.Hkv]
             sg.sgdkv_debug_enable_kernel_timing(kinds if l % every == first % every else ())
-            sg.sgdkv_score(inp["q"], inp["K"], wl.W, wl.pool, o["scores"], ws, s)
+            wsl = ws2[l % 2]
+            if l >= 2:
+                s.wait_event(pooled[l - 2])            # workspace l % 2 read by its pool
+            sg.sgdkv_score_raw(inp["q"], inp["K"], wl.W, wsl, s)
             scored[l].record(s)
             sel_stream.wait_event(scored[l])
+            sg.sgdkv_pool_raw(wsl, wl.Hkv, wl.L, wl.pool, o["scores"], sel_stream)
+            pooled[l].record(sel_stream)
             sg.sgdkv_compact(inp["K"], inp["V"], o["scores"], b, n_sink, n_recent, o["idx"],
                              o["cu"], o["ko"], o["vo"], ws_sel, sel_stream)
         done.record(sel_stream)
@@ -327,7 +335,8 @@ def run_ours(args, world, rank, local):
         return [sg.sgdkv_debug_kernel_timing(kind) for kind in range(len(KERNEL_NAMES))]
 
     def check(where):
-        st = max(sg.sgdkv_last_error(ws, stream), sg.sgdkv_last_error(ws_sel, sel_stream))
+        st = max(max(sg.sgdkv_last_error(w, stream) for w in ws2),
+                 sg.sgdkv_last_error(ws_sel, sel_stream))
         if st != sg.OK:
             raise RuntimeError(f"device-side error {where}: {sg.status_string(st)}")
 
@@ -423,8 +432,9 @@ def run_ours(args, world, rank, local):
                      "bytes_per_step": bytes_step},
         "gpu_launches": int(launches_timed),
         "schedule": "each step: budget allocation on the host, then one CUDA-graph launch of "
-                    "the step's kernels (scoring on one stream, selection + gather on a "
-                    "second inside the graph); one graph per timed step",
+                    "the step's kernels (the scoring passes on one stream, max-pool + "
+                    "selection + gather on a second inside the graph); one graph per timed "
+                    "step",
         "clocks": clk,
         "e2e": e2e,
     }

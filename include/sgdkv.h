@@ -130,6 +130,9 @@ SGDKV_API size_t sgdkv_workspace_bytes(int32_t Hq, int32_t Hkv, int64_t L, int32
  * q_win      device bf16 [Hq][W][d];  K  device bf16 [Hkv][L][d]
  * pool       odd kernel size; 1 returns the raw scores.
  * scores_out device fp32 [Hkv][L].
+ * Reproducibility: the scoring CTAs claim key tiles dynamically, and how each window row's
+ * softmax denominator is summed follows the claims, so two calls on the same input agree to
+ * within fp32 rounding (relative ~1e-6), not bit for bit.
  * Errors: INVALID_ARG, UNSUPPORTED, WORKSPACE, CUDA (launch failure).
  */
 SGDKV_API sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq, int32_t Hkv, int64_t L,
@@ -173,6 +176,26 @@ SGDKV_API sgdkv_status sgdkv_score_ex(const void* q_win, const void* K, int32_t 
                                       int64_t L, int32_t d, int32_t W, int32_t pool,
                                       uint32_t flags, const float* head_weights,
                                       float* scores_out, void* workspace, size_t ws_bytes,
+                                      void* stream);
+
+/*
+ * The two halves of sgdkv_score_ex, for callers that max-pool on another stream (the
+ * benchmark overlaps layer l's pooling and compaction with layer l+1's scoring).
+ * sgdkv_score_raw runs both scoring passes and leaves raw[h][j] (the window scores before
+ * pooling, of sgdkv_score / sgdkv_score_ex with these flags) in the workspace as partial
+ * sums; sgdkv_pool_raw max-pools them into scores_out.  In between the workspace holds the
+ * raw scores: any other call on it, sgdkv_score_raw of the next layer included, overwrites
+ * them, so a caller that overlaps layers alternates two workspaces.  sgdkv_pool_raw must
+ * get the Hkv, L and flags the raw scores were made with (the aggregation bits choose how
+ * the partial sums combine).  Arguments and errors as sgdkv_score_ex; the workspace is the
+ * one sized by sgdkv_workspace_bytes.
+ */
+SGDKV_API sgdkv_status sgdkv_score_raw(const void* q_win, const void* K, int32_t Hq, int32_t Hkv,
+                                       int64_t L, int32_t d, int32_t W, uint32_t flags,
+                                       const float* head_weights, void* workspace,
+                                       size_t ws_bytes, void* stream);
+SGDKV_API sgdkv_status sgdkv_pool_raw(const void* workspace, size_t ws_bytes, int32_t Hkv,
+                                      int64_t L, int32_t pool, uint32_t flags, float* scores_out,
                                       void* stream);
 
 /*

@@ -170,26 +170,66 @@ size_t sgdkv_workspace_bytes(int32_t Hq, int32_t Hkv, int64_t L, int32_t d, int3
   return workspace_layout(Hkv, L).total;
 }
 
+// Arguments of the scoring passes (sgdkv_score_ex, sgdkv_score_raw).
+sgdkv_status check_score_args(const void* q_win, const void* K, int32_t Hq, int32_t Hkv,
+                              int64_t L, int32_t d, int32_t W, uint32_t flags,
+                              const float* head_weights) {
+  if (!q_win || !K) return SGDKV_ERR_INVALID_ARG;
+  if (!aligned16(q_win) || !aligned16(K)) return SGDKV_ERR_INVALID_ARG;
+  if (flags & ~(SGDKV_SCORE_PROXY_QUERY | SGDKV_SCORE_AGG_MASK)) return SGDKV_ERR_INVALID_ARG;
+  const uint32_t agg = flags & SGDKV_SCORE_AGG_MASK;
+  if (agg != SGDKV_SCORE_AGG_SUM && !head_weights) return SGDKV_ERR_INVALID_ARG;
+  const sgdkv_status s = check_score_shape(Hq, Hkv, L, d, W);
+  if (s != SGDKV_OK) return s;
+  if (agg == SGDKV_SCORE_AGG_IPT_MAX && (W % 16 != 0 || W > 64 || Hq / Hkv > 8))
+    return SGDKV_ERR_UNSUPPORTED;
+  return SGDKV_OK;
+}
+
 sgdkv_status sgdkv_score_ex(const void* q_win, const void* K, int32_t Hq, int32_t Hkv, int64_t L,
                             int32_t d, int32_t W, int32_t pool, uint32_t flags,
                             const float* head_weights, float* scores_out, void* workspace,
                             size_t ws_bytes, void* stream) {
-  if (!q_win || !K || !scores_out) return SGDKV_ERR_INVALID_ARG;
-  if (!aligned16(q_win) || !aligned16(K) || !aligned16(scores_out)) return SGDKV_ERR_INVALID_ARG;
-  if (flags & ~(SGDKV_SCORE_PROXY_QUERY | SGDKV_SCORE_AGG_MASK)) return SGDKV_ERR_INVALID_ARG;
-  const uint32_t agg = flags & SGDKV_SCORE_AGG_MASK;
-  if (agg != SGDKV_SCORE_AGG_SUM && !head_weights) return SGDKV_ERR_INVALID_ARG;
-  sgdkv_status s = check_score_shape(Hq, Hkv, L, d, W);
+  if (!scores_out || !aligned16(scores_out)) return SGDKV_ERR_INVALID_ARG;
+  sgdkv_status s = check_score_args(q_win, K, Hq, Hkv, L, d, W, flags, head_weights);
   if (s != SGDKV_OK) return s;
-  if (agg == SGDKV_SCORE_AGG_IPT_MAX && (W % 16 != 0 || W > 64 || Hq / Hkv > 8))
-    return SGDKV_ERR_UNSUPPORTED;
   if ((s = check_pool(pool)) != SGDKV_OK) return s;
   if ((s = check_workspace(workspace, ws_bytes, Hkv, L)) != SGDKV_OK) return s;
   const Ws ws = workspace_view(workspace, workspace_layout(Hkv, L));
+  const uint32_t agg = flags & SGDKV_SCORE_AGG_MASK;
   return from_cuda(launch_score(static_cast<const __nv_bfloat16*>(q_win),
                                 static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, pool, flags,
                                 agg == SGDKV_SCORE_AGG_SUM ? nullptr : head_weights, scores_out,
                                 ws, static_cast<cudaStream_t>(stream)));
+}
+
+sgdkv_status sgdkv_score_raw(const void* q_win, const void* K, int32_t Hq, int32_t Hkv, int64_t L,
+                             int32_t d, int32_t W, uint32_t flags, const float* head_weights,
+                             void* workspace, size_t ws_bytes, void* stream) {
+  sgdkv_status s = check_score_args(q_win, K, Hq, Hkv, L, d, W, flags, head_weights);
+  if (s != SGDKV_OK) return s;
+  if ((s = check_workspace(workspace, ws_bytes, Hkv, L)) != SGDKV_OK) return s;
+  const Ws ws = workspace_view(workspace, workspace_layout(Hkv, L));
+  const uint32_t agg = flags & SGDKV_SCORE_AGG_MASK;
+  return from_cuda(launch_score_raw(static_cast<const __nv_bfloat16*>(q_win),
+                                    static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, flags,
+                                    agg == SGDKV_SCORE_AGG_SUM ? nullptr : head_weights, ws,
+                                    static_cast<cudaStream_t>(stream)));
+}
+
+sgdkv_status sgdkv_pool_raw(const void* workspace, size_t ws_bytes, int32_t Hkv, int64_t L,
+                            int32_t pool, uint32_t flags, float* scores_out, void* stream) {
+  if (!scores_out || !aligned16(scores_out)) return SGDKV_ERR_INVALID_ARG;
+  if (Hkv <= 0 || L <= 0) return SGDKV_ERR_INVALID_ARG;
+  if (Hkv > SGDKV_MAX_KV_HEADS || int64_t(Hkv) * L >= (int64_t(1) << 31))
+    return SGDKV_ERR_UNSUPPORTED;
+  if (flags & ~(SGDKV_SCORE_PROXY_QUERY | SGDKV_SCORE_AGG_MASK)) return SGDKV_ERR_INVALID_ARG;
+  sgdkv_status s = check_pool(pool);
+  if (s != SGDKV_OK) return s;
+  if ((s = check_workspace(const_cast<void*>(workspace), ws_bytes, Hkv, L)) != SGDKV_OK) return s;
+  const Ws ws = workspace_view(const_cast<void*>(workspace), workspace_layout(Hkv, L));
+  return from_cuda(launch_pool(ws, Hkv, L, pool, flags, scores_out,
+                               static_cast<cudaStream_t>(stream)));
 }
 
 sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq, int32_t Hkv, int64_t L,

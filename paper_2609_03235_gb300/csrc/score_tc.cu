@@ -1003,10 +1003,9 @@ int sm_count() {
 uint64_t g_score_wait_ns = 2000000000ull;
 uint32_t g_score_flags = 0;
 
-cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
-                         int64_t L, int W, int pool, uint32_t flags, const float* head_weights,
-                         float* scores_out, const Ws& ws, cudaStream_t stream) {
-  if (pool < 1 || pool / 2 > kMaxRadius) return cudaErrorInvalidValue;
+cudaError_t launch_score_raw(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
+                             int64_t L, int W, uint32_t flags, const float* head_weights,
+                             const Ws& ws, cudaStream_t stream) {
   TcParams p{};
   p.Hkv = Hkv;
   p.G = Hq / Hkv;
@@ -1068,15 +1067,32 @@ cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq,
     KernelTimer t(SGDKV_KERNEL_SCORE_PASS2, stream);
     pass2<<<grid, kThreads, smem2, stream>>>(tm_q, tm_k, p2, ws);
   }
+  note_launches(2);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pool(const Ws& ws, int Hkv, int64_t L, int pool, uint32_t flags,
+                        float* scores_out, cudaStream_t stream) {
+  if (pool < 1 || pool / 2 > kMaxRadius) return cudaErrorInvalidValue;
   {
     KernelTimer t(SGDKV_KERNEL_POOL, stream);
     const unsigned blocks = unsigned(int64_t(Hkv) * ceil_div(L, kPoolTile));
+    const bool combine_max = (flags & SGDKV_SCORE_AGG_MASK) == SGDKV_SCORE_AGG_IPT_MAX;
     maxpool_sum_kernel<<<blocks, kPoolThreads, 0, stream>>>(ws.raw, scores_out, L,
                                                             int64_t(Hkv) * L, pool / 2,
-                                                            p.agg == 1 ? 1 : 0);
+                                                            combine_max ? 1 : 0);
   }
-  note_launches(3);
+  note_launches(1);
   return cudaGetLastError();
+}
+
+cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
+                         int64_t L, int W, int pool, uint32_t flags, const float* head_weights,
+                         float* scores_out, const Ws& ws, cudaStream_t stream) {
+  if (pool < 1 || pool / 2 > kMaxRadius) return cudaErrorInvalidValue;
+  cudaError_t e = launch_score_raw(q, K, Hq, Hkv, L, W, flags, head_weights, ws, stream);
+  if (e != cudaSuccess) return e;
+  return launch_pool(ws, Hkv, L, pool, flags, scores_out, stream);
 }
 
 }  // namespace sgdkv

@@ -82,6 +82,13 @@ extern uint32_t g_score_flags;
 cudaError_t launch_score(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
                          int64_t L, int W, int pool, uint32_t flags, const float* head_weights,
                          float* scores_out, const Ws& ws, cudaStream_t stream);
+// The two halves of launch_score: both scoring passes into the raw planes of ws, and the
+// max-pool of those planes into scores_out (flags select the planes' combination).
+cudaError_t launch_score_raw(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
+                             int64_t L, int W, uint32_t flags, const float* head_weights,
+                             const Ws& ws, cudaStream_t stream);
+cudaError_t launch_pool(const Ws& ws, int Hkv, int64_t L, int pool, uint32_t flags,
+                        float* scores_out, cudaStream_t stream);
 cudaError_t launch_compact(const __nv_bfloat16* K, const __nv_bfloat16* V,
                            const float* scores, const HeadTable& ht, int32_t* indices_out,
                            int32_t* cu_out, __nv_bfloat16* K_out, __nv_bfloat16* V_out,

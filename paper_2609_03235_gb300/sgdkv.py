@@ -22,7 +22,7 @@ EXPORTED = ("sgdkv_status_string", "sgdkv_version", "sgdkv_allocate_budgets",
             "sgdkv_last_error", "sgdkv_launch_count", "sgdkv_debug_set_score_hooks",
             "sgdkv_last_cuda_error_string", "sgdkv_score_static",
             "sgdkv_debug_enable_kernel_timing", "sgdkv_debug_kernel_timing", "sgdkv_score_ex",
-            "sgdkv_mix_head_scores")
+            "sgdkv_mix_head_scores", "sgdkv_score_raw", "sgdkv_pool_raw")
 
 
 class LibraryMissing(RuntimeError):
@@ -74,6 +74,11 @@ def lib():
         L.sgdkv_score_ex.restype = ctypes.c_int
         L.sgdkv_score_ex.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, _I32, ctypes.c_uint32,
                                      _P, _P, _P, _SZ, _P]
+        L.sgdkv_score_raw.restype = ctypes.c_int
+        L.sgdkv_score_raw.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, ctypes.c_uint32, _P,
+                                      _P, _SZ, _P]
+        L.sgdkv_pool_raw.restype = ctypes.c_int
+        L.sgdkv_pool_raw.argtypes = [_P, _SZ, _I32, _I64, _I32, ctypes.c_uint32, _P, _P]
         L.sgdkv_score_static.restype = ctypes.c_int
         L.sgdkv_score_static.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, _I32, _P, _P, _P]
         L.sgdkv_debug_set_score_hooks.restype = None
@@ -168,6 +173,24 @@ def sgdkv_score(q_win, K, W: int, pool: int, scores_out, workspace, stream=None,
                               _ptr(head_weights), _ptr(scores_out), _ptr(workspace),
                               workspace.numel(), _stream(stream))
     _check(st, "sgdkv_score_ex")
+
+
+def sgdkv_score_raw(q_win, K, W: int, workspace, stream=None, flags: int = 0, head_weights=None):
+    """Both scoring passes; the raw window scores stay in the workspace for sgdkv_pool_raw."""
+    Hq, _, d = q_win.shape
+    Hkv, L, _ = K.shape
+    st = lib().sgdkv_score_raw(_ptr(q_win), _ptr(K), Hq, Hkv, L, d, W, int(flags),
+                               _ptr(head_weights), _ptr(workspace), workspace.numel(),
+                               _stream(stream))
+    _check(st, "sgdkv_score_raw")
+
+
+def sgdkv_pool_raw(workspace, Hkv: int, L: int, pool: int, scores_out, stream=None,
+                   flags: int = 0):
+    """Max-pool of the raw window scores a sgdkv_score_raw call left in the workspace."""
+    st = lib().sgdkv_pool_raw(_ptr(workspace), workspace.numel(), int(Hkv), int(L), int(pool),
+                              int(flags), _ptr(scores_out), _stream(stream))
+    _check(st, "sgdkv_pool_raw")
 
 
 def sgdkv_score_static(q_win, K, W: int, pool: int, scores_out, status_out=None, stream=None):

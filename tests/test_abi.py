@@ -159,6 +159,23 @@ def test_score_rejects_bad_args_before_device_work():
               None) == sg.ERR_INVALID_ARG
     assert ex(p, p, 28, 4, 1024, 128, 32, 7, sg.SCORE_PROXY_QUERY | sg.SCORE_AGG_IPT_MEAN, p, p,
               p, 16, None) == sg.ERR_WORKSPACE
+    # the two halves: sgdkv_score_raw checks as sgdkv_score_ex (no pool, no output)...
+    raw = L.sgdkv_score_raw
+    assert raw(None, p, 28, 4, 1024, 128, 32, 0, None, p, 1 << 30, None) == sg.ERR_INVALID_ARG
+    assert raw(p, p, 28, 4, 1024, 64, 32, 0, None, p, 1 << 30, None) == sg.ERR_UNSUPPORTED
+    assert raw(p, p, 28, 4, 1024, 128, 32, 8, None, p, 1 << 30, None) == sg.ERR_INVALID_ARG
+    assert raw(p, p, 28, 4, 1024, 128, 32, sg.SCORE_AGG_IPT_MAX, None, p, 1 << 30,
+               None) == sg.ERR_INVALID_ARG
+    assert raw(p, p, 28, 4, 1024, 128, 32, 0, None, p, 16, None) == sg.ERR_WORKSPACE
+    # ...and sgdkv_pool_raw its pool kernel, shape, flags, output and workspace
+    pr = L.sgdkv_pool_raw
+    assert pr(p, 1 << 30, 4, 1024, 6, 0, p, None) == sg.ERR_INVALID_ARG      # even pool
+    assert pr(p, 1 << 30, 0, 1024, 7, 0, p, None) == sg.ERR_INVALID_ARG      # Hkv
+    assert pr(p, 1 << 30, 4, 0, 7, 0, p, None) == sg.ERR_INVALID_ARG         # L
+    assert pr(p, 1 << 30, 4, 1024, 7, 8, p, None) == sg.ERR_INVALID_ARG      # unknown flag
+    assert pr(p, 1 << 30, 4, 1024, 7, 0, None, None) == sg.ERR_INVALID_ARG   # no output
+    assert pr(p, 1 << 30, 99, 1024, 7, 0, p, None) == sg.ERR_UNSUPPORTED     # Hkv > max
+    assert pr(p, 16, 4, 1024, 7, 0, p, None) == sg.ERR_WORKSPACE
 
 
 def test_compact_rejects_bad_budgets():

@@ -156,6 +156,45 @@ def test_ipt_aggregation_parity(dev, Hq, Hkv, L, W, mode, proxy):
     assert ok.all(), f"{(~ok).sum()} of {ok.size} off; worst {np.max(np.abs(got - exp))}"
 
 
+@pytest.mark.parametrize("flags_name", ["sum", "proxy", "ipt_max", "ipt_mean"])
+def test_score_raw_then_pool_equals_score(dev, flags_name):
+    """sgdkv_score_raw + sgdkv_pool_raw (pooling on a second stream) give what
+    sgdkv_score_ex gives (to within the run-to-run rounding of the dynamically claimed
+    row sums), and match the oracle."""
+    Hq, Hkv, L, W = 28, 4, 3000, 64
+    flags = {"sum": 0, "proxy": sg.SCORE_PROXY_QUERY, "ipt_max": sg.SCORE_AGG_IPT_MAX,
+             "ipt_mean": sg.SCORE_AGG_IPT_MEAN}[flags_name]
+    wl = synth.tiny_workload(Hq=Hq, Hkv=Hkv, d=128, L=L, W=W, n_salient=8)
+    inp = synth.tiny_inputs(wl, tag=1234)
+    q, K, _ = _upload(inp, dev)
+    w = _ipt_weights(Hq, 5)
+    hw = torch.from_numpy(w).to(dev) if flags_name.startswith("ipt") else None
+    ws_one = sg.make_workspace(Hq, Hkv, L, W, dev)
+    ws_two = sg.make_workspace(Hq, Hkv, L, W, dev)
+    one = torch.empty((Hkv, L), dtype=torch.float32, device=dev)
+    two = torch.full((Hkv, L), float("nan"), dtype=torch.float32, device=dev)
+    sg.sgdkv_score(q, K, W, 7, one, ws_one, flags=flags, head_weights=hw)
+    s_a = torch.cuda.current_stream(dev)
+    s_b = torch.cuda.Stream(dev)
+    sg.sgdkv_score_raw(q, K, W, ws_two, s_a, flags=flags, head_weights=hw)
+    ev = torch.cuda.Event()
+    ev.record(s_a)
+    s_b.wait_event(ev)
+    sg.sgdkv_pool_raw(ws_two, Hkv, L, 7, two, s_b, flags=flags)
+    torch.cuda.synchronize()
+    assert sg.sgdkv_last_error(ws_one) == sg.OK and sg.sgdkv_last_error(ws_two) == sg.OK
+    torch.testing.assert_close(two, one, rtol=1e-5, atol=1e-9)
+    if flags_name.startswith("ipt"):
+        omode = O.AGG_IPT_MAX if flags_name == "ipt_max" else O.AGG_IPT_MEAN
+        raw = O.window_scores_ipt(inp["q"], inp["K"], w, omode, causal=True)
+    else:
+        raw = O.window_scores(inp["q"], inp["K"], causal=flags_name == "sum")
+    exp = O.max_pool(raw, 7)
+    got = two.cpu().numpy()
+    ok = _within(got, exp)
+    assert ok.all(), f"{(~ok).sum()} of {ok.size} off; worst {np.max(np.abs(got - exp))}"
+
+
 def test_ipt_negative_weight_is_reported(dev):
     wl = synth.tiny_workload(Hq=14, Hkv=2, d=128, L=500, W=32, n_salient=4)
     inp = synth.tiny_inputs(wl, tag=799)
@@ -389,15 +428,16 @@ def test_compact_reads_kv_from_pinned_host_memory(dev):
 @pytest.mark.parametrize("graph", [False, True])
 def test_bench_launch_configuration_full_size(dev, graph):
     """The schedule bench.py times, at full size: consecutive layers of the 128K-context
-    Qwen2.5-7B workload, scoring on one stream and selection + gather on a second
-    (separate workspaces, layer l's compaction overlapping layer l+1's scoring), launched
-    directly or captured into a CUDA graph and replayed (bench.py's timed steps); every
-    layer end to end against the oracle."""
+    Qwen2.5-7B workload, the scoring passes on one stream (two alternating workspaces) and
+    max-pool + selection + gather on a second (layer l's pooling and compaction overlapping
+    layer l+1's scoring, layer l+2's scoring waiting for layer l's pool), launched directly
+    or captured into a CUDA graph and replayed (bench.py's timed steps); every layer end to
+    end against the oracle."""
     wl = configs.BY_NAME["c3_qwen25_7b_L128k"]
     n_sink, n_recent = configs.sink_recent_split(wl.floor)
     all_b = sg.sgdkv_allocate_budgets(synth.head_scores(wl), wl.L, wl.total_budget(0.25), wl.floor)
-    layers = [0, wl.n_layers - 1]
-    ws_a = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
+    layers = [0, 1, wl.n_layers - 1]
+    ws_a = [sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev) for _ in range(2)]
     ws_b = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
     stream_a = torch.cuda.current_stream(dev)
     stream_b = torch.cuda.Stream(dev)
@@ -419,11 +459,17 @@ def test_bench_launch_configuration_full_size(dev, graph):
         fork = torch.cuda.Event()
         fork.record(sa)
         stream_b.wait_event(fork)
-        for inp, q, K, V, b, out in runs:
-            sg.sgdkv_score(q, K, wl.W, wl.pool, out["scores"], ws_a, sa)
+        pooled = []
+        for i, (inp, q, K, V, b, out) in enumerate(runs):
+            if i >= 2:
+                sa.wait_event(pooled[i - 2])
+            sg.sgdkv_score_raw(q, K, wl.W, ws_a[i % 2], sa)
             ev = torch.cuda.Event()
             ev.record(sa)
             stream_b.wait_event(ev)
+            sg.sgdkv_pool_raw(ws_a[i % 2], wl.Hkv, wl.L, wl.pool, out["scores"], stream_b)
+            pooled.append(torch.cuda.Event())
+            pooled[-1].record(stream_b)
             sg.sgdkv_compact(K, V, out["scores"], b, n_sink, n_recent, out["indices"],
                              out["cu_seqlens"], out["K_out"], out["V_out"], ws_b, stream_b)
         done = torch.cuda.Event()
@@ -446,7 +492,7 @@ def test_bench_launch_configuration_full_size(dev, graph):
     else:
         launches(stream_a)
     torch.cuda.synchronize()
-    assert sg.sgdkv_last_error(ws_a) == sg.OK
+    assert all(sg.sgdkv_last_error(w) == sg.OK for w in ws_a)
     assert sg.sgdkv_last_error(ws_b) == sg.OK
     for inp, q, K, V, b, out in runs:
         _check_end_to_end(inp, out, b, n_sink, n_recent, wl.pool)
