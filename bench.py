@@ -43,7 +43,7 @@ def parse_args(argv=None):
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
     p.add_argument("--frac", type=float, default=0.25)
     p.add_argument("--layers", type=int, default=0, help="layers per step (0 = all)")
-    p.add_argument("--e2e-steps", type=int, default=3)
+    p.add_argument("--e2e-steps", type=int, default=4)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-child", action="store_true", help=argparse.SUPPRESS)
@@ -192,19 +192,19 @@ KERNEL_NAMES = ("score_pass1_tc", "score_pass2_tc", "maxpool_sum_kernel", "sel_c
 # DRAM traffic per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one ncu capture
 # of the 128K-context Qwen2.5-7B layer (28 query / 4 KV heads, W=64), keyed by the SHA-256 of
 # the kernel source it was taken on; a source that has changed since reads as null.
-_SCORE_SHA = "bf6ad59d9cc8036492c8592179ed3c4383e93423d2d99f2dda6040bd9bcca892"
+_SCORE_SHA = "5c16aa4044ed8d48c3cee6c9f4319da684c3d38401cb301d0f3bb14d013f6897"
 _SELECT_SHA = "390cce311b1188274ecd3021b148b6bbb18954a7a16521c4cd5ba007a67c1d4a"
 MEASURED_TRAFFIC = {
     ("score_pass1_tc", "c3_qwen25_7b_L128k"):
-        {"bytes": 134758400 + 4730368, "source": "score_tc.cu", "sha256": _SCORE_SHA},
+        {"bytes": 134759936 + 3058944, "source": "score_tc.cu", "sha256": _SCORE_SHA},
     ("score_pass2_tc", "c3_qwen25_7b_L128k"):
-        {"bytes": 135324416 + 5552128, "source": "score_tc.cu", "sha256": _SCORE_SHA},
+        {"bytes": 135347200 + 5810432, "source": "score_tc.cu", "sha256": _SCORE_SHA},
     ("maxpool_sum_kernel", "c3_qwen25_7b_L128k"):
-        {"bytes": 8398080 + 0, "source": "score_tc.cu", "sha256": _SCORE_SHA},
+        {"bytes": 8402432 + 0, "source": "score_tc.cu", "sha256": _SCORE_SHA},
     ("sel_cluster_kernel", "c3_qwen25_7b_L128k"):
-        {"bytes": 2144768 + 0, "source": "select.cu", "sha256": _SELECT_SHA},
+        {"bytes": 2144512 + 0, "source": "select.cu", "sha256": _SELECT_SHA},
     ("gather_kernel", "c3_qwen25_7b_L128k"):
-        {"bytes": 40769024 + 1928192, "source": "select.cu", "sha256": _SELECT_SHA},
+        {"bytes": 40771584 + 1879552, "source": "select.cu", "sha256": _SELECT_SHA},
 }
 
 
@@ -509,7 +509,8 @@ def run_e2e(args, wl, layers, outs, n_sink, n_recent, dev, world):
                 ho[l]["vo"].copy_(sl["vo"][:tot], non_blocking=True)
                 d2h_done[s].record(s_d2h)
 
-    step()
+    for _ in range(2):                       # warm-up: first use of the pinned pages
+        step()
     torch.cuda.synchronize(dev)
     K = args.e2e_steps
     barrier(world)
