@@ -192,7 +192,7 @@ KERNEL_NAMES = ("score_pass1_tc", "score_pass2_tc", "maxpool_sum_kernel", "sel_c
 # DRAM traffic per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one ncu capture
 # of the 128K-context Qwen2.5-7B layer (28 query / 4 KV heads, W=64), keyed by the SHA-256 of
 # the kernel source it was taken on; a source that has changed since reads as null.
-_SCORE_SHA = "5c16aa4044ed8d48c3cee6c9f4319da684c3d38401cb301d0f3bb14d013f6897"
+_SCORE_SHA = "4033adeb5b5bb66296b4361b400e39b65ceb3603305303573f06460552e5ed16"
 _SELECT_SHA = "390cce311b1188274ecd3021b148b6bbb18954a7a16521c4cd5ba007a67c1d4a"
 MEASURED_TRAFFIC = {
     ("score_pass1_tc", "c3_qwen25_7b_L128k"):

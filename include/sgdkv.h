@@ -199,6 +199,28 @@ SGDKV_API sgdkv_status sgdkv_pool_raw(const void* workspace, size_t ws_bytes, in
                                       void* stream);
 
 /*
+ * sgdkv_score_raw's two passes as separate calls (steps a2 and a3 of the scoring: Section
+ * 3.3's softmax over the keys needs every window row's normaliser before any key's sum).
+ * sgdkv_window_stats: window logits t_rj = q_r . k_j / sqrt(d) and, per window row r, the
+ * online (max, sum of exp) over the keys the row sees, kept in the workspace.
+ * sgdkv_window_sums: recomputes the logits and sums exp(t_rj - lse_r) over the window rows
+ * (and the GQA group, with the flags' aggregation) per key, from the statistics a
+ * sgdkv_window_stats call with the same arguments left in the same workspace; the raw
+ * scores then wait there for sgdkv_pool_raw.  The workspace holds the statistics in
+ * between: a caller that overlaps layers (one layer's sums beside the next layer's
+ * statistics) gives each layer in flight its own workspace.  Arguments and errors as
+ * sgdkv_score_raw.
+ */
+SGDKV_API sgdkv_status sgdkv_window_stats(const void* q_win, const void* K, int32_t Hq,
+                                          int32_t Hkv, int64_t L, int32_t d, int32_t W,
+                                          uint32_t flags, const float* head_weights,
+                                          void* workspace, size_t ws_bytes, void* stream);
+SGDKV_API sgdkv_status sgdkv_window_sums(const void* q_win, const void* K, int32_t Hq,
+                                         int32_t Hkv, int64_t L, int32_t d, int32_t W,
+                                         uint32_t flags, const float* head_weights,
+                                         void* workspace, size_t ws_bytes, void* stream);
+
+/*
  * sgdkv_score without a workspace argument, for callers that cannot allocate device
  * memory (for example code running where the allocator is owned by someone else, or a
  * plugin that may only receive tensors).  No counterpart in the paper: the computation

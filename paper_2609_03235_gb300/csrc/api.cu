@@ -217,6 +217,36 @@ sgdkv_status sgdkv_score_raw(const void* q_win, const void* K, int32_t Hq, int32
                                     static_cast<cudaStream_t>(stream)));
 }
 
+sgdkv_status sgdkv_window_stats(const void* q_win, const void* K, int32_t Hq, int32_t Hkv,
+                                int64_t L, int32_t d, int32_t W, uint32_t flags,
+                                const float* head_weights, void* workspace, size_t ws_bytes,
+                                void* stream) {
+  sgdkv_status s = check_score_args(q_win, K, Hq, Hkv, L, d, W, flags, head_weights);
+  if (s != SGDKV_OK) return s;
+  if ((s = check_workspace(workspace, ws_bytes, Hkv, L)) != SGDKV_OK) return s;
+  const Ws ws = workspace_view(workspace, workspace_layout(Hkv, L));
+  const uint32_t agg = flags & SGDKV_SCORE_AGG_MASK;
+  return from_cuda(launch_passes(static_cast<const __nv_bfloat16*>(q_win),
+                                 static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, flags,
+                                 agg == SGDKV_SCORE_AGG_SUM ? nullptr : head_weights, ws,
+                                 static_cast<cudaStream_t>(stream), 1u));
+}
+
+sgdkv_status sgdkv_window_sums(const void* q_win, const void* K, int32_t Hq, int32_t Hkv,
+                               int64_t L, int32_t d, int32_t W, uint32_t flags,
+                               const float* head_weights, void* workspace, size_t ws_bytes,
+                               void* stream) {
+  sgdkv_status s = check_score_args(q_win, K, Hq, Hkv, L, d, W, flags, head_weights);
+  if (s != SGDKV_OK) return s;
+  if ((s = check_workspace(workspace, ws_bytes, Hkv, L)) != SGDKV_OK) return s;
+  const Ws ws = workspace_view(workspace, workspace_layout(Hkv, L));
+  const uint32_t agg = flags & SGDKV_SCORE_AGG_MASK;
+  return from_cuda(launch_passes(static_cast<const __nv_bfloat16*>(q_win),
+                                 static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, flags,
+                                 agg == SGDKV_SCORE_AGG_SUM ? nullptr : head_weights, ws,
+                                 static_cast<cudaStream_t>(stream), 2u));
+}
+
 sgdkv_status sgdkv_pool_raw(const void* workspace, size_t ws_bytes, int32_t Hkv, int64_t L,
                             int32_t pool, uint32_t flags, float* scores_out, void* stream) {
   if (!scores_out || !aligned16(scores_out)) return SGDKV_ERR_INVALID_ARG;

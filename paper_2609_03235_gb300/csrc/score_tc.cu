@@ -1003,9 +1003,9 @@ int sm_count() {
 uint64_t g_score_wait_ns = 2000000000ull;
 uint32_t g_score_flags = 0;
 
-cudaError_t launch_score_raw(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
-                             int64_t L, int W, uint32_t flags, const float* head_weights,
-                             const Ws& ws, cudaStream_t stream) {
+cudaError_t launch_passes(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
+                          int64_t L, int W, uint32_t flags, const float* head_weights,
+                          const Ws& ws, cudaStream_t stream, unsigned passes) {
   TcParams p{};
   p.Hkv = Hkv;
   p.G = Hq / Hkv;
@@ -1059,16 +1059,23 @@ cudaError_t launch_score_raw(const __nv_bfloat16* q, const __nv_bfloat16* K, int
                                 int(smem2))) != cudaSuccess)
     return e;
   const int grid = Hkv * p.cph;
-  {
+  if (passes & 1u) {
     KernelTimer t(SGDKV_KERNEL_SCORE_PASS1, stream);
     pass1<<<grid, kThreads, smem1, stream>>>(tm_q, tm_k, p1, ws);
+    note_launches(1);
   }
-  {
+  if (passes & 2u) {
     KernelTimer t(SGDKV_KERNEL_SCORE_PASS2, stream);
     pass2<<<grid, kThreads, smem2, stream>>>(tm_q, tm_k, p2, ws);
+    note_launches(1);
   }
-  note_launches(2);
   return cudaGetLastError();
+}
+
+cudaError_t launch_score_raw(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
+                             int64_t L, int W, uint32_t flags, const float* head_weights,
+                             const Ws& ws, cudaStream_t stream) {
+  return launch_passes(q, K, Hq, Hkv, L, W, flags, head_weights, ws, stream, 3u);
 }
 
 cudaError_t launch_pool(const Ws& ws, int Hkv, int64_t L, int pool, uint32_t flags,

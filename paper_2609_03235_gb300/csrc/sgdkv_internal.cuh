@@ -89,6 +89,11 @@ cudaError_t launch_score_raw(const __nv_bfloat16* q, const __nv_bfloat16* K, int
                              const Ws& ws, cudaStream_t stream);
 cudaError_t launch_pool(const Ws& ws, int Hkv, int64_t L, int pool, uint32_t flags,
                         float* scores_out, cudaStream_t stream);
+// launch_score_raw's passes one at a time: bit 0 pass 1 (window-row statistics into the
+// workspace), bit 1 pass 2 (the window sums, reading those statistics).
+cudaError_t launch_passes(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
+                          int64_t L, int W, uint32_t flags, const float* head_weights,
+                          const Ws& ws, cudaStream_t stream, unsigned passes);
 cudaError_t launch_compact(const __nv_bfloat16* K, const __nv_bfloat16* V,
                            const float* scores, const HeadTable& ht, int32_t* indices_out,
                            int32_t* cu_out, __nv_bfloat16* K_out, __nv_bfloat16* V_out,

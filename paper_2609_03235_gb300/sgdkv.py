@@ -22,7 +22,8 @@ EXPORTED = ("sgdkv_status_string", "sgdkv_version", "sgdkv_allocate_budgets",
             "sgdkv_last_error", "sgdkv_launch_count", "sgdkv_debug_set_score_hooks",
             "sgdkv_last_cuda_error_string", "sgdkv_score_static",
             "sgdkv_debug_enable_kernel_timing", "sgdkv_debug_kernel_timing", "sgdkv_score_ex",
-            "sgdkv_mix_head_scores", "sgdkv_score_raw", "sgdkv_pool_raw")
+            "sgdkv_mix_head_scores", "sgdkv_score_raw", "sgdkv_pool_raw",
+            "sgdkv_window_stats", "sgdkv_window_sums")
 
 
 class LibraryMissing(RuntimeError):
@@ -77,6 +78,9 @@ def lib():
         L.sgdkv_score_raw.restype = ctypes.c_int
         L.sgdkv_score_raw.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, ctypes.c_uint32, _P,
                                       _P, _SZ, _P]
+        for fn in (L.sgdkv_window_stats, L.sgdkv_window_sums):
+            fn.restype = ctypes.c_int
+            fn.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, ctypes.c_uint32, _P, _P, _SZ, _P]
         L.sgdkv_pool_raw.restype = ctypes.c_int
         L.sgdkv_pool_raw.argtypes = [_P, _SZ, _I32, _I64, _I32, ctypes.c_uint32, _P, _P]
         L.sgdkv_score_static.restype = ctypes.c_int
@@ -183,6 +187,28 @@ def sgdkv_score_raw(q_win, K, W: int, workspace, stream=None, flags: int = 0, he
                                _ptr(head_weights), _ptr(workspace), workspace.numel(),
                                _stream(stream))
     _check(st, "sgdkv_score_raw")
+
+
+def _window_pass(fn, name, q_win, K, W, workspace, stream, flags, head_weights):
+    Hq, _, d = q_win.shape
+    Hkv, L, _ = K.shape
+    st = fn(_ptr(q_win), _ptr(K), Hq, Hkv, L, d, W, int(flags), _ptr(head_weights),
+            _ptr(workspace), workspace.numel(), _stream(stream))
+    _check(st, name)
+
+
+def sgdkv_window_stats(q_win, K, W: int, workspace, stream=None, flags: int = 0,
+                       head_weights=None):
+    """Pass 1 of the scoring: per-window-row softmax statistics into the workspace."""
+    _window_pass(lib().sgdkv_window_stats, "sgdkv_window_stats", q_win, K, W, workspace, stream,
+                 flags, head_weights)
+
+
+def sgdkv_window_sums(q_win, K, W: int, workspace, stream=None, flags: int = 0,
+                      head_weights=None):
+    """Pass 2 of the scoring: the raw window scores, from sgdkv_window_stats' statistics."""
+    _window_pass(lib().sgdkv_window_sums, "sgdkv_window_sums", q_win, K, W, workspace, stream,
+                 flags, head_weights)
 
 
 def sgdkv_pool_raw(workspace, Hkv: int, L: int, pool: int, scores_out, stream=None,

@@ -167,6 +167,12 @@ def test_score_rejects_bad_args_before_device_work():
     assert raw(p, p, 28, 4, 1024, 128, 32, sg.SCORE_AGG_IPT_MAX, None, p, 1 << 30,
                None) == sg.ERR_INVALID_ARG
     assert raw(p, p, 28, 4, 1024, 128, 32, 0, None, p, 16, None) == sg.ERR_WORKSPACE
+    # the two passes one at a time check the same
+    for fn in (L.sgdkv_window_stats, L.sgdkv_window_sums):
+        assert fn(None, p, 28, 4, 1024, 128, 32, 0, None, p, 1 << 30, None) == sg.ERR_INVALID_ARG
+        assert fn(p, p, 28, 4, 1024, 64, 32, 0, None, p, 1 << 30, None) == sg.ERR_UNSUPPORTED
+        assert fn(p, p, 28, 4, 1024, 128, 32, 8, None, p, 1 << 30, None) == sg.ERR_INVALID_ARG
+        assert fn(p, p, 28, 4, 1024, 128, 32, 0, None, p, 16, None) == sg.ERR_WORKSPACE
     # ...and sgdkv_pool_raw its pool kernel, shape, flags, output and workspace
     pr = L.sgdkv_pool_raw
     assert pr(p, 1 << 30, 4, 1024, 6, 0, p, None) == sg.ERR_INVALID_ARG      # even pool

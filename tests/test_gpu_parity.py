@@ -195,6 +195,44 @@ def test_score_raw_then_pool_equals_score(dev, flags_name):
     assert ok.all(), f"{(~ok).sum()} of {ok.size} off; worst {np.max(np.abs(got - exp))}"
 
 
+@pytest.mark.parametrize("flags_name", ["sum", "proxy", "ipt_max"])
+def test_window_stats_then_sums_two_layers_in_flight(dev, flags_name):
+    """sgdkv_window_stats / sgdkv_window_sums / sgdkv_pool_raw as separate calls, two
+    layers in flight on two streams (layer 1's statistics beside layer 0's sums, one
+    workspace each), against the oracle."""
+    Hq, Hkv, L, W = 28, 4, 3000, 64
+    flags = {"sum": 0, "proxy": sg.SCORE_PROXY_QUERY, "ipt_max": sg.SCORE_AGG_IPT_MAX}[flags_name]
+    wl = synth.tiny_workload(Hq=Hq, Hkv=Hkv, d=128, L=L, W=W, n_salient=8)
+    w = _ipt_weights(Hq, 11)
+    hw = torch.from_numpy(w).to(dev) if flags_name == "ipt_max" else None
+    s_a, s_b = torch.cuda.current_stream(dev), torch.cuda.Stream(dev)
+    layers = []
+    for tag in (501, 502):
+        inp = synth.tiny_inputs(wl, tag=tag)
+        q, K, _ = _upload(inp, dev)
+        layers.append((inp, q, K, sg.make_workspace(Hq, Hkv, L, W, dev),
+                       torch.full((Hkv, L), float("nan"), dtype=torch.float32, device=dev)))
+    torch.cuda.synchronize()
+    for inp, q, K, ws, out in layers:
+        sg.sgdkv_window_stats(q, K, W, ws, s_a, flags=flags, head_weights=hw)
+        ev = torch.cuda.Event()
+        ev.record(s_a)
+        s_b.wait_event(ev)
+        sg.sgdkv_window_sums(q, K, W, ws, s_b, flags=flags, head_weights=hw)
+        sg.sgdkv_pool_raw(ws, Hkv, L, 7, out, s_b, flags=flags)
+    torch.cuda.synchronize()
+    for inp, q, K, ws, out in layers:
+        assert sg.sgdkv_last_error(ws) == sg.OK
+        if flags_name == "ipt_max":
+            raw = O.window_scores_ipt(inp["q"], inp["K"], w, O.AGG_IPT_MAX, causal=True)
+        else:
+            raw = O.window_scores(inp["q"], inp["K"], causal=flags_name == "sum")
+        exp = O.max_pool(raw, 7)
+        got = out.cpu().numpy()
+        ok = _within(got, exp)
+        assert ok.all(), f"{(~ok).sum()} of {ok.size} off; worst {np.max(np.abs(got - exp))}"
+
+
 def test_ipt_negative_weight_is_reported(dev):
     wl = synth.tiny_workload(Hq=14, Hkv=2, d=128, L=500, W=32, n_salient=4)
     inp = synth.tiny_inputs(wl, tag=799)
