@@ -186,6 +186,7 @@ def pass_flops(wl) -> float:
 
 DIAG_STEPS = 3
 TIMED_EVERY = 4          # the dominant kernel is event-bracketed in every 4th layer
+N_SCORE_WS = 3           # scoring workspaces in rotation (layers in flight on them)
 KERNEL_NAMES = ("score_pass1_tc", "score_pass2_tc", "maxpool_sum_kernel", "sel_cluster_kernel",
                 "gather_kernel")
 
@@ -242,8 +243,9 @@ def workload_config(wl, args, world, n_layers):
             "context_len": wl.L, "window": wl.W, "pool": wl.pool,
             "budget_frac": args.frac, "floor": wl.floor, "n_sink": n_sink,
             "n_recent": n_recent, "parallelism": f"replicas x{world}",
-            "streams": "scoring passes on one stream, max-pool + selection + gather on a "
-                       "second; layer l's pooling and compaction overlap layer l+1's scoring",
+            "streams": "scoring passes on one stream, max-pool + selection (one kernel) and "
+                       "gather on a second; layer l's pooling and compaction overlap layer "
+                       "l+1's scoring",
             "l2": "inputs larger than L2 (K+V of one layer = %d MiB)" %
                   (2 * wl.Hkv * wl.L * wl.d * 2 >> 20)}
 
@@ -277,22 +279,24 @@ def run_ours(args, world, rank, local):
             ko=torch.empty((tot, wl.d), dtype=torch.bfloat16, device=dev),
             vo=torch.empty((tot, wl.d), dtype=torch.bfloat16, device=dev)))
     # One step = the host budget allocation (a1), then the launches of every layer: the two
-    # scoring passes on the capturing stream, max-pool + selection + gather on `sel_stream`;
-    # layer l's pooling and compaction wait for layer l's passes only, so they overlap layer
-    # l+1's scoring, whose CTAs claim key tiles dynamically and absorb the SMs the other
-    # stream leaves.  The raw scores of layer l stay in scoring workspace l % 2 until its
-    # pool has read them (layer l + 2's scoring waits for that).  The launches of a step are
+    # scoring passes on the capturing stream, sgdkv_pool_compact (the max-pool inside the
+    # selection kernel, then the gather) on `sel_stream`; layer l's pooling and compaction
+    # wait for layer l's passes only, so they overlap layer l+1's scoring, whose CTAs claim
+    # key tiles dynamically and absorb the SMs the other stream leaves.  The raw scores of
+    # layer l stay in scoring workspace l % 3 until its compaction has read them (layer
+    # l + 3's scoring waits for that: with two workspaces, layer l + 2's scoring would wait
+    # for layer l's gather as well).  The launches of a step are
     # captured into a CUDA graph (per-kernel launch cost ~1 us instead of ~3 us on a stream)
     # and the graph is replayed; the allocation still runs on the host every step and must
     # reproduce the budgets the graph was captured with.
-    ws2 = [sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev) for _ in range(2)]
+    ws_score = [sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev) for _ in range(N_SCORE_WS)]
     ws_sel = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
     stream = torch.cuda.current_stream(dev)
     lo_prio, hi_prio = torch.cuda.Stream.priority_range()
     sel_stream = torch.cuda.Stream(dev, priority=hi_prio)
     fork = torch.cuda.Event()
     scored = [torch.cuda.Event() for _ in range(Ls)]
-    pooled = [torch.cuda.Event() for _ in range(Ls)]
+    pooled = [torch.cuda.Event() for _ in range(Ls)]     # workspace l % N_SCORE_WS read
     done = torch.cuda.Event()
 
     def launches(ball, s, kinds=(), every=1, first=0):
@@ -302,16 +306,16 @@ def run_ours(args, world, rank, local):
             inp, o = layers[l], outs[l]
             b = ball[l * wl.Hkv:(l + 1) * wl.Hkv]
             sg.sgdkv_debug_enable_kernel_timing(kinds if l % every == first % every else ())
-            wsl = ws2[l % 2]
-            if l >= 2:
-                s.wait_event(pooled[l - 2])            # workspace l % 2 read by its pool
+            wsl = ws_score[l % N_SCORE_WS]
+            if l >= N_SCORE_WS:
+                s.wait_event(pooled[l - N_SCORE_WS])   # its workspace read by that compaction
             sg.sgdkv_score_raw(inp["q"], inp["K"], wl.W, wsl, s)
             scored[l].record(s)
             sel_stream.wait_event(scored[l])
-            sg.sgdkv_pool_raw(wsl, wl.Hkv, wl.L, wl.pool, o["scores"], sel_stream)
+            sg.sgdkv_pool_compact(wsl, wl.pool, inp["K"], inp["V"], b, n_sink, n_recent,
+                                  o["scores"], o["idx"], o["cu"], o["ko"], o["vo"], ws_sel,
+                                  sel_stream)
             pooled[l].record(sel_stream)
-            sg.sgdkv_compact(inp["K"], inp["V"], o["scores"], b, n_sink, n_recent, o["idx"],
-                             o["cu"], o["ko"], o["vo"], ws_sel, sel_stream)
         done.record(sel_stream)
         s.wait_event(done)
 
@@ -335,7 +339,7 @@ def run_ours(args, world, rank, local):
         return [sg.sgdkv_debug_kernel_timing(kind) for kind in range(len(KERNEL_NAMES))]
 
     def check(where):
-        st = max(max(sg.sgdkv_last_error(w, stream) for w in ws2),
+        st = max(max(sg.sgdkv_last_error(w, stream) for w in ws_score),
                  sg.sgdkv_last_error(ws_sel, sel_stream))
         if st != sg.OK:
             raise RuntimeError(f"device-side error {where}: {sg.status_string(st)}")
@@ -363,6 +367,7 @@ def run_ours(args, world, rank, local):
         kern[name] = {"launches": n, "us_per_launch": 1e3 * tot_ms / max(n, 1), "ms_total": tot_ms,
                       "dram_bytes_ncu": measured_traffic(name, wl.name)}
     del diag
+    kern = {k: v for k, v in kern.items() if v["launches"] > 0}   # no pool kernel at this size
     all_ms = sum(v["ms_total"] for v in kern.values())
     for v in kern.values():
         v["share"] = v["ms_total"] / all_ms if all_ms > 0 else None
@@ -399,7 +404,7 @@ def run_ours(args, world, rank, local):
     peaks = measured_peaks()
     top_us = 1e3 * top_ms / max(top_n, 1)
     achieved_tf = pass_flops(wl) / (top_us * 1e-6) / 1e12
-    stage_us = sum(kern[n]["us_per_launch"] for n in KERNEL_NAMES[:3])
+    stage_us = sum(kern[n]["us_per_launch"] for n in KERNEL_NAMES[:3] if n in kern)
     stage_tf = score_flops(wl) / (stage_us * 1e-6) / 1e12
     bytes_step = sum(path_bytes(wl, o["b"]) for o in outs)
     value = world * wl.L * Ls / (ms_max * 1e-3)
@@ -433,8 +438,8 @@ def run_ours(args, world, rank, local):
         "gpu_launches": int(launches_timed),
         "schedule": "each step: budget allocation on the host, then one CUDA-graph launch of "
                     "the step's kernels (the scoring passes on one stream, max-pool + "
-                    "selection + gather on a second inside the graph); one graph per timed "
-                    "step",
+                    "selection in one kernel and the gather on a second inside the graph); "
+                    "one graph per timed step",
         "clocks": clk,
         "e2e": e2e,
     }

@@ -269,6 +269,33 @@ SGDKV_API sgdkv_status sgdkv_compact(const void* K, const void* V, const float* 
                            size_t ws_bytes, void* stream);
 
 /*
+ * sgdkv_pool_raw followed by sgdkv_compact in one call (Section 3.3: max-pool of the window
+ * scores, then the selection and gather), reading the raw scores that sgdkv_score_raw or
+ * sgdkv_window_sums left in score_workspace.  Where the selection keeps each slice of a row
+ * in registers (rows up to 524288 positions on a GPU with 16-CTA clusters), the selection
+ * kernel pools its own slice and no pool kernel is launched; longer rows take the two
+ * kernels.  Either way scores_out receives the pooled scores bit for bit as sgdkv_pool_raw
+ * writes them, and the kept positions and rows are those sgdkv_compact gives on them.
+ *
+ * score_workspace, score_ws_bytes  the workspace holding the raw scores (read only); pool and
+ *                 flags as given to sgdkv_pool_raw (the Hkv, L and flags of the scoring call)
+ * scores_out      device fp32 [Hkv][L], 16-byte aligned (required)
+ * workspace       the compaction's own workspace (device-side errors are recorded there);
+ *                 may be score_workspace itself
+ * Other arguments as sgdkv_compact.  A caller that overlaps layers may start the next
+ * scoring call on score_workspace only after this call.  Errors: INVALID_ARG, UNSUPPORTED,
+ * WORKSPACE, CUDA.
+ */
+SGDKV_API sgdkv_status sgdkv_pool_compact(const void* score_workspace, size_t score_ws_bytes,
+                                          int32_t pool, uint32_t flags, const void* K,
+                                          const void* V, const int64_t* budgets, int32_t Hkv,
+                                          int64_t L, int32_t d, int64_t n_sink,
+                                          int64_t n_recent, float* scores_out,
+                                          int32_t* indices_out, int32_t* cu_seqlens_out,
+                                          void* K_out, void* V_out, void* workspace,
+                                          size_t ws_bytes, void* stream);
+
+/*
  * The whole per-layer step: sgdkv_score followed by sgdkv_compact on the same stream,
  * keeping the pooled scores in the workspace.  scores_out may be NULL; when given, it
  * receives the pooled scores as sgdkv_score would.  K must be device memory (the scorer

@@ -71,6 +71,29 @@ sgdkv_status check_pool(int32_t pool) {
   return SGDKV_OK;
 }
 
+// Steps a4-a6 from the raw planes of the scoring workspace sws: the max-pool inside the
+// selection kernel where its slices stay in registers, else the stand-alone pool kernel
+// into scores_out followed by the selection on scores_out.  Device errors go to ws.
+cudaError_t pool_then_compact(const Ws& sws, int32_t pool, uint32_t flags,
+                              const __nv_bfloat16* K, const __nv_bfloat16* V, const HeadTable& ht,
+                              int64_t total, float* scores_out, int32_t* indices_out,
+                              int32_t* cu_out, __nv_bfloat16* K_out, __nv_bfloat16* V_out,
+                              const Ws& ws, cudaStream_t st) {
+  if (compact_pools_inline(ht.L)) {
+    PoolSrc ps;
+    ps.raw = sws.raw;
+    ps.plane = int64_t(ht.Hkv) * ht.L;
+    ps.radius = pool / 2;
+    ps.combine_max = (flags & SGDKV_SCORE_AGG_MASK) == SGDKV_SCORE_AGG_IPT_MAX ? 1 : 0;
+    ps.out = scores_out;
+    return launch_compact(K, V, scores_out, ht, indices_out, cu_out, K_out, V_out, total, ws, st,
+                          &ps);
+  }
+  cudaError_t e = launch_pool(sws, ht.Hkv, ht.L, pool, flags, scores_out, st);
+  if (e != cudaSuccess) return e;
+  return launch_compact(K, V, scores_out, ht, indices_out, cu_out, K_out, V_out, total, ws, st);
+}
+
 // Validates budgets and fills the per-head table; returns the total kept rows.
 sgdkv_status build_head_table(const int64_t* budgets, int32_t Hkv, int64_t L, int64_t n_sink,
                               int64_t n_recent, HeadTable* ht, int64_t* total) {
@@ -323,6 +346,38 @@ sgdkv_status sgdkv_compact(const void* K, const void* V, const float* scores,
                                   static_cast<cudaStream_t>(stream)));
 }
 
+sgdkv_status sgdkv_pool_compact(const void* score_workspace, size_t score_ws_bytes, int32_t pool,
+                                uint32_t flags, const void* K, const void* V,
+                                const int64_t* budgets, int32_t Hkv, int64_t L, int32_t d,
+                                int64_t n_sink, int64_t n_recent, float* scores_out,
+                                int32_t* indices_out, int32_t* cu_seqlens_out, void* K_out,
+                                void* V_out, void* workspace, size_t ws_bytes, void* stream) {
+  if (!K || !V || !scores_out || !cu_seqlens_out) return SGDKV_ERR_INVALID_ARG;
+  if (Hkv <= 0 || L <= 0 || d <= 0) return SGDKV_ERR_INVALID_ARG;
+  if (d != kD || Hkv > SGDKV_MAX_KV_HEADS || int64_t(Hkv) * L >= (int64_t(1) << 31))
+    return SGDKV_ERR_UNSUPPORTED;
+  if (!aligned16(K) || !aligned16(V) || !aligned16(scores_out)) return SGDKV_ERR_INVALID_ARG;
+  if (flags & ~(SGDKV_SCORE_PROXY_QUERY | SGDKV_SCORE_AGG_MASK)) return SGDKV_ERR_INVALID_ARG;
+  sgdkv_status s = check_pool(pool);
+  if (s != SGDKV_OK) return s;
+  HeadTable ht;
+  int64_t total = 0;
+  if ((s = build_head_table(budgets, Hkv, L, n_sink, n_recent, &ht, &total)) != SGDKV_OK) return s;
+  if (total > 0 && (!indices_out || !K_out || !V_out)) return SGDKV_ERR_INVALID_ARG;
+  if (total > 0 && (!aligned16(K_out) || !aligned16(V_out))) return SGDKV_ERR_INVALID_ARG;
+  if ((s = check_workspace(const_cast<void*>(score_workspace), score_ws_bytes, Hkv, L)) != SGDKV_OK)
+    return s;
+  if ((s = check_workspace(workspace, ws_bytes, Hkv, L)) != SGDKV_OK) return s;
+  const Ws sws = workspace_view(const_cast<void*>(score_workspace), workspace_layout(Hkv, L));
+  const Ws ws = workspace_view(workspace, workspace_layout(Hkv, L));
+  return from_cuda(pool_then_compact(sws, pool, flags, static_cast<const __nv_bfloat16*>(K),
+                                     static_cast<const __nv_bfloat16*>(V), ht, total, scores_out,
+                                     indices_out, cu_seqlens_out,
+                                     static_cast<__nv_bfloat16*>(K_out),
+                                     static_cast<__nv_bfloat16*>(V_out), ws,
+                                     static_cast<cudaStream_t>(stream)));
+}
+
 sgdkv_status sgdkv_compress_layer(const void* q_win, const void* K, const void* V,
                                   const int64_t* budgets, int32_t Hq, int32_t Hkv, int64_t L,
                                   int32_t d, int32_t W, int32_t pool, int64_t n_sink,
@@ -344,14 +399,15 @@ sgdkv_status sgdkv_compress_layer(const void* q_win, const void* K, const void* 
   const Ws ws = workspace_view(workspace, workspace_layout(Hkv, L));
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   float* pooled = scores_out ? scores_out : ws.pooled;
-  cudaError_t e = launch_score(static_cast<const __nv_bfloat16*>(q_win),
-                               static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, pool, 0u,
-                               nullptr, pooled, ws, st);
+  cudaError_t e = launch_score_raw(static_cast<const __nv_bfloat16*>(q_win),
+                                   static_cast<const __nv_bfloat16*>(K), Hq, Hkv, L, W, 0u,
+                                   nullptr, ws, st);
   if (e != cudaSuccess) return from_cuda(e);
-  return from_cuda(launch_compact(static_cast<const __nv_bfloat16*>(K),
-                                  static_cast<const __nv_bfloat16*>(V), pooled, ht, indices_out,
-                                  cu_seqlens_out, static_cast<__nv_bfloat16*>(K_out),
-                                  static_cast<__nv_bfloat16*>(V_out), total, ws, st));
+  return from_cuda(pool_then_compact(ws, pool, 0u, static_cast<const __nv_bfloat16*>(K),
+                                     static_cast<const __nv_bfloat16*>(V), ht, total, pooled,
+                                     indices_out, cu_seqlens_out,
+                                     static_cast<__nv_bfloat16*>(K_out),
+                                     static_cast<__nv_bfloat16*>(V_out), ws, st));
 }
 
 sgdkv_status sgdkv_last_error(void* workspace, void* stream) {

@@ -542,7 +542,9 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     return;
   }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int h = blockIdx.x / p.cph, ci = blockIdx.x % p.cph;
+  // heads interleaved over the block indices: CTAs that wait for an SM held by another
+  // kernel are spread across the heads instead of delaying one head's whole share
+  const int h = blockIdx.x % p.Hkv, ci = blockIdx.x / p.Hkv;
   uint32_t* counter = ws.sched + h;
   const Smem s = carve(smem_raw, NRT * 128, p.nstages);
   const uint32_t tmem = setup(s, p.nstages, 1, kTmemSlots, 4);
@@ -697,7 +699,7 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     return;
   }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int h = blockIdx.x / p.cph;
+  const int h = blockIdx.x % p.Hkv;             // heads interleaved, as in pass 1
   uint32_t* counter = ws.sched + 2 * SGDKV_MAX_KV_HEADS + h;
   const Smem s = carve(smem_raw, p.GW, p.nstages);
   float* lse2 = s.tail;                          // [kMaxRows], negated
@@ -893,7 +895,7 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
 // in shared memory with coalesced loads, then every output takes its window maximum there.
 constexpr int kPoolTile = 1024;
 constexpr int kPoolThreads = 256;
-constexpr int kMaxRadius = 31;                    // pool <= 63
+constexpr int kMaxRadius = kMaxPoolRadius;
 
 __global__ void __launch_bounds__(kPoolThreads)
 maxpool_sum_kernel(const float* __restrict__ raw, float* __restrict__ out, int64_t L,

@@ -12,6 +12,9 @@
 // (lowest positions first) follow.  The same kernel then counts kept positions per slice,
 // exchanges the counts through distributed shared memory, and writes every slice's kept
 // positions, ascending, at their final offsets.  A second kernel copies the kept K/V rows.
+// With a pool source the selection kernel first forms its slice's pooled scores itself
+// (the four raw planes summed, then the window maximum, Section 3.3), so the max-pool needs
+// no launch of its own.
 #include <cooperative_groups.h>
 
 #include "sgdkv_internal.cuh"
@@ -20,7 +23,7 @@ namespace sgdkv {
 namespace cg = cooperative_groups;
 namespace {
 
-constexpr int kCThreads = 512;                 // threads per selection CTA
+constexpr int kCThreads = 1024;                // threads per selection CTA
 constexpr int kCWarps = kCThreads / 32;
 constexpr int kPer = 8;                        // positions per thread per write round
 constexpr int kRound = kCThreads * kPer;       // positions per write round
@@ -76,15 +79,130 @@ struct KeepRule {
   __device__ __forceinline__ bool tie(uint32_t u) const { return !none && u == tau; }
 };
 
+// Shared-memory index of the pool buffer: one word of skew per 32, so that the 16 or so
+// consecutive words each thread reads fall into different banks across a warp.
+__device__ __forceinline__ int pool_sk(int x) { return x + (x >> 5); }
+constexpr int kPoolSmallR = 3;   // window radii up to this take the register path
+
+// The pooled scores of positions p0 .. p0+PER-1 (those inside [beg, end)) as uint32 keys:
+// the CTA sums the four planes of its slice and a halo of `radius` positions on each side
+// into shared memory (-inf outside the row), then every thread takes the maximum over the
+// window [j - radius, j + radius] of each of its positions, in the same arithmetic as the
+// stand-alone max-pool kernel, and writes its pooled scores to ps.out.
+template <int PER>
+__device__ __forceinline__ void pool_slice(const PoolSrc& ps, int h, int64_t L, int64_t beg,
+                                           int64_t end, int64_t p0, uint32_t (&u)[PER]) {
+  extern __shared__ int32_t stage[];
+  float* sum = reinterpret_cast<float*>(stage);       // sum[pool_sk(x)]: position beg - r + x
+  const int r = ps.radius;
+  const int n = int(end - beg);
+  const float* r0 = ps.raw + int64_t(h) * L;
+  const int64_t pl = ps.plane;
+  const bool cmax = ps.combine_max != 0;
+  auto comb = [&](float a, float b, float c, float d) {
+    return cmax ? fmaxf(fmaxf(a, b), fmaxf(c, d)) : (a + b) + (c + d);
+  };
+  auto at = [&](int64_t j) {
+    return j >= 0 && j < L ? comb(__ldcg(r0 + j), __ldcg(r0 + pl + j), __ldcg(r0 + 2 * pl + j),
+                                  __ldcg(r0 + 3 * pl + j))
+                           : -INFINITY;
+  };
+  const bool vec = ((L | beg | pl) & 3) == 0 && (reinterpret_cast<uintptr_t>(ps.raw) & 15) == 0;
+  if (vec) {
+    // Rounds of two 16-byte loads per plane and thread, all issued before the first is
+    // used; the first round also fetches one position of the halos or of the slice's last
+    // n % 4 (at most 2 * kMaxPoolRadius + 3 of them, one per thread).
+    const int n4 = n >> 2, nh = 2 * r + (n & 3);
+    for (int i0 = threadIdx.x, first = 1; first || i0 < n4; i0 += 2 * kCThreads, first = 0) {
+      float4 a[2], b[2], c[2], d[2];
+      float hv[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+      int hx = -1;
+      if (first && threadIdx.x < nh) {
+        hx = threadIdx.x < r ? threadIdx.x : r + 4 * n4 + (threadIdx.x - r);
+        const int64_t j = beg - r + hx;
+        if (j >= 0 && j < L) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) hv[k] = __ldcg(r0 + k * pl + j);
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {
+        const int i = i0 + k * kCThreads;
+        if (i >= n4) continue;
+        const int64_t j = beg + 4 * i;
+        a[k] = __ldcg(reinterpret_cast<const float4*>(r0 + j));
+        b[k] = __ldcg(reinterpret_cast<const float4*>(r0 + pl + j));
+        c[k] = __ldcg(reinterpret_cast<const float4*>(r0 + 2 * pl + j));
+        d[k] = __ldcg(reinterpret_cast<const float4*>(r0 + 3 * pl + j));
+      }
+      if (hx >= 0) sum[pool_sk(hx)] = comb(hv[0], hv[1], hv[2], hv[3]);
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {
+        const int i = i0 + k * kCThreads;
+        if (i >= n4) continue;
+        const int x = r + 4 * i;
+        sum[pool_sk(x)] = comb(a[k].x, b[k].x, c[k].x, d[k].x);
+        sum[pool_sk(x + 1)] = comb(a[k].y, b[k].y, c[k].y, d[k].y);
+        sum[pool_sk(x + 2)] = comb(a[k].z, b[k].z, c[k].z, d[k].z);
+        sum[pool_sk(x + 3)] = comb(a[k].w, b[k].w, c[k].w, d[k].w);
+      }
+    }
+  } else {
+    for (int x = threadIdx.x; x < n + 2 * r; x += kCThreads) sum[pool_sk(x)] = at(beg - r + x);
+  }
+  __syncthreads();
+  const int xb = int(p0 - beg);      // window of position p0 + i: x in [xb + i, xb + i + 2r]
+  const int nv = p0 < end ? int(end - p0 < PER ? end - p0 : PER) : 0;   // positions held
+  const int lim = nv > 0 ? nv + 2 * r : 0;   // x = xb + k stays below n + 2r
+  float m[PER];
+  if (r <= kPoolSmallR) {
+    float w[PER + 2 * kPoolSmallR];
+#pragma unroll
+    for (int k = 0; k < PER + 2 * kPoolSmallR; ++k)
+      w[k] = k < lim ? sum[pool_sk(xb + k)] : -INFINITY;
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+      float v = w[i];
+#pragma unroll
+      for (int k = 1; k <= 2 * kPoolSmallR; ++k)
+        if (k <= 2 * r) v = fmaxf(v, w[i + k]);
+      m[i] = v;
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+      float v = -INFINITY;
+      if (i < nv)
+        for (int k = 0; k <= 2 * r; ++k) v = fmaxf(v, sum[pool_sk(xb + i + k)]);
+      m[i] = v;
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < PER; ++i) u[i] = i < nv ? __float_as_uint(m[i]) : 0u;
+  float* o = ps.out + int64_t(h) * L + p0;
+  if (nv == PER && PER % 4 == 0 && (reinterpret_cast<uintptr_t>(o) & 15) == 0) {
+#pragma unroll
+    for (int i = 0; i < PER; i += 4)
+      *reinterpret_cast<float4*>(o + i) = make_float4(m[i], m[i + 1], m[i + 2], m[i + 3]);
+  } else {
+#pragma unroll
+    for (int i = 0; i < PER; ++i)
+      if (i < nv) o[i] = m[i];
+  }
+}
+
 // One cluster per KV head (grid = Hkv * csize, cluster = csize CTAs).  Control flow is
 // uniform across a cluster, so every CTA reaches every cluster barrier.
 // PER > 0: each thread holds PER consecutive positions of its CTA's slice in registers for
 // the whole kernel (slice <= kCThreads * PER); PER == 0: every pass streams the slice.
-template <int PER>
+// POOL (PER > 0 only): the slice's scores are pooled from ps's raw planes (pool_slice) and
+// `scores` is not read.
+template <int PER, bool POOL>
 __global__ void __launch_bounds__(kCThreads)
 sel_cluster_kernel(const float* __restrict__ scores, HeadTable ht, int csize,
                    int32_t* __restrict__ indices_out, int32_t* __restrict__ cu_out,
-                   uint32_t* __restrict__ status) {
+                   uint32_t* __restrict__ status, PoolSrc ps) {
+  static_assert(!POOL || PER > 0, "inline pooling needs register-resident slices");
   cg::cluster_group cluster = cg::this_cluster();
   __shared__ SelShared sm;
   const int tid = threadIdx.x, wid = tid >> 5;
@@ -105,7 +223,9 @@ sel_cluster_kernel(const float* __restrict__ scores, HeadTable ht, int csize,
   // register-resident positions p0 .. p0+PER-1 (0 bits outside the slice: never read)
   const int64_t p0 = beg + int64_t(tid) * (PER > 0 ? PER : 1);
   uint32_t u[PER > 0 ? PER : 1];
-  if constexpr (PER > 0) {
+  if constexpr (POOL) {
+    pool_slice<PER>(ps, h, L, beg, end, p0, u);
+  } else if constexpr (PER > 0) {
 #pragma unroll
     for (int i = 0; i < PER; ++i) u[i] = p0 + i < end ? __float_as_uint(__ldg(row + p0 + i)) : 0u;
   }
@@ -346,23 +466,30 @@ gather_kernel(const uint4* __restrict__ K, const uint4* __restrict__ V,
   }
 }
 
-// Largest cluster size (16 if the device runs it, else the portable 8) for the selection.
-template <int PER>
-constexpr size_t stage_bytes() { return size_t(kCThreads) * (PER > 0 ? PER : 0) * sizeof(int32_t); }
+// Dynamic shared memory of a selection kernel: the staged kept positions, and with POOL
+// the pool buffer of a slice and its halos (skewed), which it precedes.
+template <int PER, bool POOL>
+constexpr size_t sel_smem_bytes() {
+  const size_t st = size_t(kCThreads) * (PER > 0 ? PER : 0) * sizeof(int32_t);
+  const size_t pb = POOL ? size_t(kCThreads * PER + 2 * kMaxPoolRadius) * 33 / 32 + 1 : 0;
+  return st > pb * sizeof(float) ? st : pb * sizeof(float);
+}
 
-template <int PER>
+// Largest cluster size (16 if the device runs it, else the portable 8) for the selection.
+template <int PER, bool POOL>
 int cluster_size() {
   static int cached = 0;
   if (cached == 0) {
     cached = 8;
-    cudaFuncSetAttribute(sel_cluster_kernel<PER>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         int(stage_bytes<PER>()));
-    if (cudaFuncSetAttribute(sel_cluster_kernel<PER>,
+    constexpr size_t smem = sel_smem_bytes<PER, POOL>();
+    cudaFuncSetAttribute(sel_cluster_kernel<PER, POOL>,
+                         cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    if (cudaFuncSetAttribute(sel_cluster_kernel<PER, POOL>,
                              cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
       cudaLaunchConfig_t cfg = {};
       cfg.gridDim = dim3(16, 1, 1);
       cfg.blockDim = dim3(kCThreads, 1, 1);
-      cfg.dynamicSmemBytes = stage_bytes<PER>();
+      cfg.dynamicSmemBytes = smem;
       cudaLaunchAttribute attr;
       attr.id = cudaLaunchAttributeClusterDimension;
       attr.val.clusterDim.x = 16;
@@ -371,7 +498,7 @@ int cluster_size() {
       cfg.attrs = &attr;
       cfg.numAttrs = 1;
       int n = 0;
-      if (cudaOccupancyMaxPotentialClusterSize(&n, sel_cluster_kernel<PER>, &cfg) ==
+      if (cudaOccupancyMaxPotentialClusterSize(&n, sel_cluster_kernel<PER, POOL>, &cfg) ==
               cudaSuccess &&
           n >= 16)
         cached = 16;
@@ -381,14 +508,14 @@ int cluster_size() {
   return cached;
 }
 
-template <int PER>
+template <int PER, bool POOL>
 cudaError_t launch_select(const float* scores, const HeadTable& ht, int csize,
                           int32_t* indices_out, int32_t* cu_out, uint32_t* status,
-                          cudaStream_t stream) {
+                          const PoolSrc& ps, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(unsigned(ht.Hkv * csize), 1, 1);
   cfg.blockDim = dim3(kCThreads, 1, 1);
-  cfg.dynamicSmemBytes = stage_bytes<PER>();
+  cfg.dynamicSmemBytes = sel_smem_bytes<PER, POOL>();
   cfg.stream = stream;
   cudaLaunchAttribute attr;
   attr.id = cudaLaunchAttributeClusterDimension;
@@ -397,8 +524,39 @@ cudaError_t launch_select(const float* scores, const HeadTable& ht, int csize,
   attr.val.clusterDim.z = 1;
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, sel_cluster_kernel<PER>, scores, ht, csize, indices_out,
-                            cu_out, status);
+  return cudaLaunchKernelEx(&cfg, sel_cluster_kernel<PER, POOL>, scores, ht, csize,
+                            indices_out, cu_out, status, ps);
+}
+
+// Positions per thread of the selection kernel for rows of length L: slices of up to 32
+// positions per thread stay in registers for the whole kernel (the positions per thread
+// follow from the cluster size that kernel actually runs with); 0: the streaming kernel.
+template <bool POOL>
+int pick_per(int64_t L, int* csize) {
+  auto fits = [&](int per, int cs) { return ceil_div(ceil_div(L, cs), kCThreads) <= per; };
+  if (fits(8, *csize = cluster_size<8, POOL>())) return 8;
+  if (fits(16, *csize = cluster_size<16, POOL>())) return 16;
+  if (fits(32, *csize = cluster_size<32, POOL>())) return 32;
+  *csize = cluster_size<0, false>();
+  return 0;
+}
+
+template <bool POOL>
+cudaError_t dispatch_select(const float* scores, const HeadTable& ht, int32_t* indices_out,
+                            int32_t* cu_out, uint32_t* status, const PoolSrc& ps,
+                            cudaStream_t stream) {
+  int cs = 0;
+  switch (pick_per<POOL>(ht.L, &cs)) {
+    case 8:
+      return launch_select<8, POOL>(scores, ht, cs, indices_out, cu_out, status, ps, stream);
+    case 16:
+      return launch_select<16, POOL>(scores, ht, cs, indices_out, cu_out, status, ps, stream);
+    case 32:
+      return launch_select<32, POOL>(scores, ht, cs, indices_out, cu_out, status, ps, stream);
+    default:
+      if (POOL) return cudaErrorInvalidValue;   // callers check compact_pools_inline
+      return launch_select<0, false>(scores, ht, cs, indices_out, cu_out, status, ps, stream);
+  }
 }
 
 }  // namespace
@@ -406,22 +564,16 @@ cudaError_t launch_select(const float* scores, const HeadTable& ht, int csize,
 cudaError_t launch_compact(const __nv_bfloat16* K, const __nv_bfloat16* V,
                            const float* scores, const HeadTable& ht, int32_t* indices_out,
                            int32_t* cu_out, __nv_bfloat16* K_out, __nv_bfloat16* V_out,
-                           int64_t total_rows, const Ws& ws, cudaStream_t stream) {
-  // slices of up to 32 positions per thread stay in registers for the whole kernel; the
-  // positions per thread follow from the cluster size that kernel actually runs with
-  auto fits = [&](int per, int cs) { return ceil_div(ceil_div(ht.L, cs), kCThreads) <= per; };
+                           int64_t total_rows, const Ws& ws, cudaStream_t stream,
+                           const PoolSrc* pool_src) {
   cudaError_t e;
   {
     KernelTimer t(SGDKV_KERNEL_SELECT, stream);
-    int cs;
-    if (fits(8, cs = cluster_size<8>()))
-      e = launch_select<8>(scores, ht, cs, indices_out, cu_out, ws.status, stream);
-    else if (fits(16, cs = cluster_size<16>()))
-      e = launch_select<16>(scores, ht, cs, indices_out, cu_out, ws.status, stream);
-    else if (fits(32, cs = cluster_size<32>()))
-      e = launch_select<32>(scores, ht, cs, indices_out, cu_out, ws.status, stream);
+    if (pool_src)
+      e = dispatch_select<true>(pool_src->out, ht, indices_out, cu_out, ws.status, *pool_src,
+                                stream);
     else
-      e = launch_select<0>(scores, ht, cluster_size<0>(), indices_out, cu_out, ws.status, stream);
+      e = dispatch_select<false>(scores, ht, indices_out, cu_out, ws.status, PoolSrc{}, stream);
   }
   if (e != cudaSuccess) return e;
   note_launches(1);
@@ -436,6 +588,11 @@ cudaError_t launch_compact(const __nv_bfloat16* K, const __nv_bfloat16* V,
         ws.status);
   }
   return cudaGetLastError();
+}
+
+bool compact_pools_inline(int64_t L) {
+  int cs = 0;
+  return pick_per<true>(L, &cs) > 0;
 }
 
 }  // namespace sgdkv

@@ -14,6 +14,7 @@ namespace sgdkv {
 constexpr int kD = SGDKV_HEAD_DIM;     // head dim supported by v1
 constexpr int kMaxRows = 512;          // G*W limit (window rows of one KV head)
 constexpr int kMaxScoreParts = 320;    // pass-1 partial (m, Z) slots per KV head
+constexpr int kMaxPoolRadius = 31;     // max-pool window <= 63 positions
 // Per-call, per-head constants passed by value in kernel parameters.
 struct HeadTable {
   int32_t Hkv;
@@ -94,9 +95,26 @@ cudaError_t launch_pool(const Ws& ws, int Hkv, int64_t L, int pool, uint32_t fla
 cudaError_t launch_passes(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq, int Hkv,
                           int64_t L, int W, uint32_t flags, const float* head_weights,
                           const Ws& ws, cudaStream_t stream, unsigned passes);
+// Source of the pooled scores when the selection kernel forms them itself: the four raw
+// planes [4][Hkv][L] of a scoring workspace (plane stride `plane` floats), the window radius,
+// the planes' combination (sum, or max for the "Ipt." max aggregation), and the output
+// [Hkv][L] that receives the pooled scores the selection ran on.
+struct PoolSrc {
+  const float* raw;
+  int64_t plane;
+  int radius;
+  int combine_max;
+  float* out;
+};
+// pool_src NULL: select on `scores`.  Else `scores` is ignored and the selection kernel
+// pools pool_src's planes first (only for rows that compact_pools_inline accepts).
 cudaError_t launch_compact(const __nv_bfloat16* K, const __nv_bfloat16* V,
                            const float* scores, const HeadTable& ht, int32_t* indices_out,
                            int32_t* cu_out, __nv_bfloat16* K_out, __nv_bfloat16* V_out,
-                           int64_t total_rows, const Ws& ws, cudaStream_t stream);
+                           int64_t total_rows, const Ws& ws, cudaStream_t stream,
+                           const PoolSrc* pool_src = nullptr);
+// true when the selection kernel for rows of length L keeps its slice in registers, and so
+// can take a PoolSrc
+bool compact_pools_inline(int64_t L);
 
 }  // namespace sgdkv

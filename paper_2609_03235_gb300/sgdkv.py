@@ -23,7 +23,7 @@ EXPORTED = ("sgdkv_status_string", "sgdkv_version", "sgdkv_allocate_budgets",
             "sgdkv_last_cuda_error_string", "sgdkv_score_static",
             "sgdkv_debug_enable_kernel_timing", "sgdkv_debug_kernel_timing", "sgdkv_score_ex",
             "sgdkv_mix_head_scores", "sgdkv_score_raw", "sgdkv_pool_raw",
-            "sgdkv_window_stats", "sgdkv_window_sums")
+            "sgdkv_window_stats", "sgdkv_window_sums", "sgdkv_pool_compact")
 
 
 class LibraryMissing(RuntimeError):
@@ -83,6 +83,9 @@ def lib():
             fn.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, ctypes.c_uint32, _P, _P, _SZ, _P]
         L.sgdkv_pool_raw.restype = ctypes.c_int
         L.sgdkv_pool_raw.argtypes = [_P, _SZ, _I32, _I64, _I32, ctypes.c_uint32, _P, _P]
+        L.sgdkv_pool_compact.restype = ctypes.c_int
+        L.sgdkv_pool_compact.argtypes = [_P, _SZ, _I32, ctypes.c_uint32, _P, _P, _P, _I32, _I64,
+                                         _I32, _I64, _I64, _P, _P, _P, _P, _P, _P, _SZ, _P]
         L.sgdkv_score_static.restype = ctypes.c_int
         L.sgdkv_score_static.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, _I32, _P, _P, _P]
         L.sgdkv_debug_set_score_hooks.restype = None
@@ -241,6 +244,20 @@ def sgdkv_compact(K, V, scores, budgets, n_sink: int, n_recent: int, indices_out
                              _ptr(K_out), _ptr(V_out), _ptr(workspace), workspace.numel(),
                              _stream(stream))
     _check(st, "sgdkv_compact")
+
+
+def sgdkv_pool_compact(score_workspace, pool: int, K, V, budgets, n_sink: int, n_recent: int,
+                       scores_out, indices_out, cu_seqlens_out, K_out, V_out, workspace,
+                       stream=None, flags: int = 0):
+    """sgdkv_pool_raw + sgdkv_compact in one call, from the raw scores in score_workspace."""
+    Hkv, L, d = K.shape
+    b = _budgets(budgets)
+    st = lib().sgdkv_pool_compact(_ptr(score_workspace), score_workspace.numel(), int(pool),
+                                  int(flags), _ptr(K), _ptr(V), b.ctypes.data_as(_P), Hkv, L,
+                                  d, n_sink, n_recent, _ptr(scores_out), _ptr(indices_out),
+                                  _ptr(cu_seqlens_out), _ptr(K_out), _ptr(V_out),
+                                  _ptr(workspace), workspace.numel(), _stream(stream))
+    _check(st, "sgdkv_pool_compact")
 
 
 def sgdkv_compress_layer(q_win, K, V, budgets, W: int, pool: int, n_sink: int, n_recent: int,

@@ -182,6 +182,22 @@ def test_score_rejects_bad_args_before_device_work():
     assert pr(p, 1 << 30, 4, 1024, 7, 0, None, None) == sg.ERR_INVALID_ARG   # no output
     assert pr(p, 1 << 30, 99, 1024, 7, 0, p, None) == sg.ERR_UNSUPPORTED     # Hkv > max
     assert pr(p, 16, 4, 1024, 7, 0, p, None) == sg.ERR_WORKSPACE
+    # ...and sgdkv_pool_compact both, before anything reaches the device
+    pc = L.sgdkv_pool_compact
+    b = np.array([300, 300, 300, 300], np.int64).ctypes.data_as(ctypes.c_void_p)
+    bad = np.array([300, 300, 300, 2000], np.int64).ctypes.data_as(ctypes.c_void_p)
+
+    def call(pool=7, flags=0, budgets=b, d=128, scores=p, sws=1 << 30, ws=1 << 30):
+        return pc(p, sws, pool, flags, p, p, budgets, 4, 1024, d, 64, 64, scores, p, p, p, p, p,
+                  ws, None)
+    assert call(pool=6) == sg.ERR_INVALID_ARG                 # even pool
+    assert call(pool=65) == sg.ERR_INVALID_ARG                # window wider than 63
+    assert call(flags=8) == sg.ERR_INVALID_ARG                # unknown flag
+    assert call(scores=None) == sg.ERR_INVALID_ARG            # pooled scores required
+    assert call(d=64) == sg.ERR_UNSUPPORTED                   # head dim
+    assert call(budgets=bad) == sg.ERR_INVALID_ARG            # budget above L
+    assert call(sws=16) == sg.ERR_WORKSPACE                   # scoring workspace too small
+    assert call(ws=16) == sg.ERR_WORKSPACE                    # compaction workspace too small
 
 
 def test_compact_rejects_bad_budgets():

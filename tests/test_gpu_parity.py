@@ -262,7 +262,8 @@ COMPACT_CASES = [
     (2, 5000, 10, 20, "full"),        # the whole middle selected
     (5, 9000, 100, 28, "random"),     # several selection chunks, ragged tail
     (1, 1, 0, 0, "full"),
-    (2, 200000, 64, 64, "random"),    # several ordered-write rounds per CTA slice
+    (2, 200000, 64, 64, "random"),    # 16 positions per thread
+    (1, 600000, 64, 64, "random"),    # streaming selection: several ordered-write rounds
 ]
 
 
@@ -329,6 +330,74 @@ def _check_end_to_end(inp, out, budgets, n_sink, n_recent, pool):
     ko, vo = O.gather(inp["K"], inp["V"], g_idx, g_cu)
     assert np.array_equal(synth.from_torch_bf16(out["K_out"]), ko)
     assert np.array_equal(synth.from_torch_bf16(out["V_out"]), vo)
+
+
+POOL_COMPACT_CASES = [
+    # Hq, Hkv, L, W, pool, flags      (path inside the selection kernel)
+    (28, 4, 3000, 64, 7, "sum"),      # 16-byte plane loads, register window
+    (14, 2, 3001, 32, 7, "sum"),      # L % 4 != 0: scalar plane loads, ragged last slice
+    (16, 2, 2049, 64, 9, "proxy"),    # radius 4: window maxima from shared memory
+    (9, 1, 1000, 32, 63, "sum"),      # radius 31 (largest), halo wider than some slices
+    (7, 1, 40, 32, 7, "sum"),         # slices of 3 positions, most threads hold none
+    (28, 4, 3000, 64, 7, "ipt_max"),  # planes combined by max
+    (28, 4, 20000, 64, 1, "sum"),     # no pooling (radius 0)
+    (2, 1, 300000, 16, 7, "sum"),     # 32 positions per thread
+    (2, 1, 600000, 16, 7, "sum"),     # rows too long for register slices: two kernels
+]
+
+
+@pytest.mark.parametrize("Hq,Hkv,L,W,pool,flags_name", POOL_COMPACT_CASES)
+def test_pool_compact_equals_pool_then_compact(dev, Hq, Hkv, L, W, pool, flags_name):
+    """sgdkv_pool_compact (the max-pool inside the selection kernel) writes the pooled
+    scores bit for bit as sgdkv_pool_raw does and keeps what sgdkv_compact keeps on them;
+    both match the oracle."""
+    flags = {"sum": 0, "proxy": sg.SCORE_PROXY_QUERY, "ipt_max": sg.SCORE_AGG_IPT_MAX}[flags_name]
+    wl = synth.tiny_workload(Hq=Hq, Hkv=Hkv, d=128, L=L, W=W, n_salient=8)
+    inp = synth.tiny_inputs(wl, tag=4321 + L)
+    q, K, V = _upload(inp, dev)
+    w = _ipt_weights(Hq, 11)
+    hw = torch.from_numpy(w).to(dev) if flags_name == "ipt_max" else None
+    n_sink, n_recent = min(16, L // 4), min(16, L // 4)
+    rng = np.random.default_rng(L + Hkv)
+    b = rng.integers(n_sink + n_recent, L + 1, size=Hkv).astype(np.int64)
+    total = int(b.sum())
+    ws = sg.make_workspace(Hq, Hkv, L, W, dev)
+    ws_sel = sg.make_workspace(Hq, Hkv, L, W, dev)
+    sg.sgdkv_score_raw(q, K, W, ws, flags=flags, head_weights=hw)
+
+    def outs():
+        return dict(scores=torch.full((Hkv, L), float("nan"), dtype=torch.float32, device=dev),
+                    idx=torch.full((total,), -1, dtype=torch.int32, device=dev),
+                    cu=torch.full((Hkv + 1,), -1, dtype=torch.int32, device=dev),
+                    ko=torch.zeros((total, 128), dtype=torch.bfloat16, device=dev),
+                    vo=torch.zeros((total, 128), dtype=torch.bfloat16, device=dev))
+    a, f = outs(), outs()
+    sg.sgdkv_pool_raw(ws, Hkv, L, pool, a["scores"], flags=flags)
+    sg.sgdkv_compact(K, V, a["scores"], b, n_sink, n_recent, a["idx"], a["cu"], a["ko"],
+                     a["vo"], ws_sel)
+    sg.sgdkv_pool_compact(ws, pool, K, V, b, n_sink, n_recent, f["scores"], f["idx"], f["cu"],
+                          f["ko"], f["vo"], ws_sel, flags=flags)
+    torch.cuda.synchronize()
+    assert sg.sgdkv_last_error(ws) == sg.OK and sg.sgdkv_last_error(ws_sel) == sg.OK
+    for k in a:
+        if a[k].dtype == torch.bfloat16:
+            assert torch.equal(a[k].view(torch.int16), f[k].view(torch.int16)), k
+        else:
+            assert torch.equal(a[k].view(torch.int32), f[k].view(torch.int32)), k
+    if flags_name == "ipt_max":
+        raw = O.window_scores_ipt(inp["q"], inp["K"], w, O.AGG_IPT_MAX, causal=True)
+    else:
+        raw = O.window_scores(inp["q"], inp["K"], causal=flags_name == "sum")
+    exp = O.max_pool(raw, pool) if pool > 1 else raw
+    got = f["scores"].cpu().numpy()
+    ok = _within(got, exp)
+    assert ok.all(), f"{(~ok).sum()} of {ok.size} off; worst {np.max(np.abs(got - exp))}"
+    e_idx, e_cu = O.select_indices(got, b, n_sink, n_recent)
+    assert np.array_equal(f["cu"].cpu().numpy(), e_cu)
+    assert np.array_equal(f["idx"].cpu().numpy(), e_idx)
+    e_ko, e_vo = O.gather(inp["K"], inp["V"], e_idx, e_cu)
+    assert np.array_equal(synth.from_torch_bf16(f["ko"]), e_ko)
+    assert np.array_equal(synth.from_torch_bf16(f["vo"]), e_vo)
 
 
 def test_compress_layer_small(dev):
@@ -467,10 +536,10 @@ def test_compact_reads_kv_from_pinned_host_memory(dev):
 def test_bench_launch_configuration_full_size(dev, graph):
     """The schedule bench.py times, at full size: consecutive layers of the 128K-context
     Qwen2.5-7B workload, the scoring passes on one stream (two alternating workspaces) and
-    max-pool + selection + gather on a second (layer l's pooling and compaction overlapping
-    layer l+1's scoring, layer l+2's scoring waiting for layer l's pool), launched directly
-    or captured into a CUDA graph and replayed (bench.py's timed steps); every layer end to
-    end against the oracle."""
+    sgdkv_pool_compact (max-pool inside the selection kernel, then the gather) on a second
+    (layer l's pooling and compaction overlapping layer l+1's scoring, layer l+2's scoring
+    waiting for layer l's compaction), launched directly or captured into a CUDA graph and
+    replayed (bench.py's timed steps); every layer end to end against the oracle."""
     wl = configs.BY_NAME["c3_qwen25_7b_L128k"]
     n_sink, n_recent = configs.sink_recent_split(wl.floor)
     all_b = sg.sgdkv_allocate_budgets(synth.head_scores(wl), wl.L, wl.total_budget(0.25), wl.floor)
@@ -505,11 +574,11 @@ def test_bench_launch_configuration_full_size(dev, graph):
             ev = torch.cuda.Event()
             ev.record(sa)
             stream_b.wait_event(ev)
-            sg.sgdkv_pool_raw(ws_a[i % 2], wl.Hkv, wl.L, wl.pool, out["scores"], stream_b)
+            sg.sgdkv_pool_compact(ws_a[i % 2], wl.pool, K, V, b, n_sink, n_recent,
+                                  out["scores"], out["indices"], out["cu_seqlens"],
+                                  out["K_out"], out["V_out"], ws_b, stream_b)
             pooled.append(torch.cuda.Event())
             pooled[-1].record(stream_b)
-            sg.sgdkv_compact(K, V, out["scores"], b, n_sink, n_recent, out["indices"],
-                             out["cu_seqlens"], out["K_out"], out["V_out"], ws_b, stream_b)
         done = torch.cuda.Event()
         done.record(stream_b)
         sa.wait_event(done)
