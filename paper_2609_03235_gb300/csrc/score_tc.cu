@@ -166,6 +166,21 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
       : "memory");
 }
+// The same with an L2 cache policy (createpolicy) for the copied lines.
+__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap* map, int x,
+                                                 int y, uint32_t bar, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      ".L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(policy)
+      : "memory");
+}
+// L2 policy of lines read for the last time: first to be evicted.
+__device__ __forceinline__ uint64_t l2_evict_first() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
 
 // Shared-memory matrix descriptor (K-major operand, 128-byte swizzle, rows of 128 bytes in
 // 8-row atoms of 1024 bytes: the layout a TMA box {64 bf16, rows} with SWIZZLE_128B writes),
@@ -394,9 +409,12 @@ __device__ __forceinline__ void teardown(uint32_t tmem) {
 // TMA producer (one thread): Q rows of head h once, then key tiles of head h claimed one
 // at a time from the head's counter (shared by the head's CTAs; the next claim is made while
 // the current tile's stage is awaited) until none are left; the stage after the last one
-// carries tile id -1 and no data.
+// carries tile id -1 and no data.  second (pass 2): pass 2 reads the keys pass 1 has just
+// read, so it takes a head's tiles from the last one down, starting on the tiles pass 1
+// loaded last, which are still in L2, and loads them evict-first (nothing reads them after
+// pass 2), so that its misses do not push out the tiles it has yet to reach.
 __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMap* tm_k,
-                        const TcParams& p, int h, uint32_t* counter, bool load_q,
+                        const TcParams& p, int h, uint32_t* counter, bool load_q, bool second,
                         uint32_t* status) {
   volatile int* ab = s.abort_flag;
   if (load_q) {
@@ -408,12 +426,15 @@ __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMa
   }
   int issued[kMaxStages];
   for (int i = 0; i < kMaxStages; ++i) issued[i] = 0;
+  const uint64_t k_policy = second ? l2_evict_first() : 0;
   uint32_t next = atomicAdd(counter, 1u);       // the next claim overlaps the stage wait
   for (int n = 0;; ++n) {
     const int st = n % p.nstages;
     const int use = n / p.nstages;
-    const uint32_t tile = next;
-    if (tile < uint32_t(p.T)) next = atomicAdd(counter, 1u);
+    const uint32_t claim = next;
+    const uint32_t tile =
+        second && claim < uint32_t(p.T) ? uint32_t(p.T) - 1u - claim : claim;
+    if (claim < uint32_t(p.T)) next = atomicAdd(counter, 1u);
     if (!bwait(bar_kempty(s, st), (use & 1) ^ 1, ab, p.wait_ns, status)) break;
     if (tile >= uint32_t(p.T)) {
       s.stile[st] = -1;
@@ -423,9 +444,13 @@ __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMa
     s.stile[st] = int(tile);
     mbar_expect_tx(bar_kfull(s, st), kStageBytes);
     const int row = int(int64_t(h) * p.L + int64_t(tile) * kTileKeys);
-    for (int c = 0; c < 2; ++c)
-      tma_load_2d(smem_u32(s.k + st * kStageBytes + c * kHalfBytes), tm_k, 64 * c, row,
-                  bar_kfull(s, st));
+    for (int c = 0; c < 2; ++c) {
+      const uint32_t dst = smem_u32(s.k + st * kStageBytes + c * kHalfBytes);
+      if (second)
+        tma_load_2d_hint(dst, tm_k, 64 * c, row, bar_kfull(s, st), k_policy);
+      else
+        tma_load_2d(dst, tm_k, 64 * c, row, bar_kfull(s, st));
+    }
     issued[st] = use + 1;
   }
   if (*ab) {
@@ -551,7 +576,7 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   volatile int* ab = s.abort_flag;
 
   if (warp == kProducerWarp) {
-    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, counter, true, ws.status);
+    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, counter, true, false, ws.status);
   } else if (warp == kMmaWarp) {
     const uint32_t leader = elect_one();
     const uint32_t idesc = idesc_bf16(128, kTileKeys);
@@ -709,7 +734,7 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   const int nn = p.GW / nch;                     // MMA N
 
   if (warp == kProducerWarp) {
-    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, counter, true, ws.status);
+    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, counter, true, true, ws.status);
   } else if (warp == kMmaWarp) {
     const uint32_t leader = elect_one();
     const uint32_t idesc = idesc_bf16(128, nn);
