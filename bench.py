@@ -194,7 +194,7 @@ KERNEL_NAMES = ("score_pass1_tc", "score_pass2_tc", "maxpool_sum_kernel", "sel_c
 # of the 128K-context Qwen2.5-7B layer (28 query / 4 KV heads, W=64), keyed by the SHA-256 of
 # the kernel source it was taken on; a source that has changed since reads as null.
 _SCORE_SHA = "e7936773fbe7ce70c3b7e0ac5c4f49450047f96a7e980040dce6593adc033e28"
-_SELECT_SHA = "dcc236d8a397c206b7a04b6ecca05a007013356c85d26a140be211a41e1af468"
+_SELECT_SHA = "95ec997644c3fdfdf93a0671515bfdb607f37f72d5ada6e648711d459661f0be"
 MEASURED_TRAFFIC = {
     ("score_pass1_tc", "c3_qwen25_7b_L128k"):
         {"bytes": 134755072 + 3629568, "source": "score_tc.cu", "sha256": _SCORE_SHA},

@@ -459,10 +459,12 @@ gather_kernel(const uint4* __restrict__ K, const uint4* __restrict__ V,
       continue;
     }
     const int64_t src = (int64_t(lo) * ht.L + j) * 16 + part;
-    const uint4 kv = __ldg(K + src);
-    const uint4 vv = __ldg(V + src);
-    Ko[o * 16 + part] = kv;
-    Vo[o * 16 + part] = vv;
+    // rows read and written once: streaming (evict-first) loads and stores, so that the copy
+    // does not push out of L2 the key tiles pass 2 of the next layer is about to re-read
+    const uint4 kv = __ldcs(K + src);
+    const uint4 vv = __ldcs(V + src);
+    __stcs(Ko + o * 16 + part, kv);
+    __stcs(Vo + o * 16 + part, vv);
   }
 }
 
