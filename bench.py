@@ -203,8 +203,7 @@ MEASURED_TRAFFIC = {
     ("sel_cluster_kernel", "c3_qwen25_7b_L128k"):
         {"bytes": 8444416 + 0, "source": "select.cu", "sha256": _SELECT_SHA},
     ("gather_kernel", "c3_qwen25_7b_L128k"):
-        {"bytes": 40768256 + 1885952, "source": "select.cu",
-         "sha256": "dcc236d8a397c206b7a04b6ecca05a007013356c85d26a140be211a41e1af468"},
+        {"bytes": 40768768 + 1776896, "source": "select.cu", "sha256": _SELECT_SHA},
 }
 
 
