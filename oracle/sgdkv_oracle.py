@@ -34,6 +34,11 @@ Steps and the passages they follow (SGD-KV, "Summarization Guided KV Cache Compr
   broken by the lower position.  Output positions ascending per head, with cu_seqlens.
 * ``gather``: keep the selected K/V rows per KV head (Appendix, "allocations occur
   before repeating the KV values": one cache per KV head), concatenated head by head.
+* ``decode_attention``: what generation computes over the compressed cache (Section 3.3:
+  the retained tokens are the heads' history; Appendix, Configuration: the cache is kept
+  per KV head, before the values are repeated for the query heads of a GQA group): for
+  each query head and new token, softmax(q . k / sqrt(d)) over its KV head's kept rows,
+  times those rows' values.  A head with no kept row gives zeros (the paper is silent).
 
 Parity pins for every function live in ``tests/test_oracle_*.py``.
 """
@@ -332,6 +337,35 @@ def gather(K, V, indices, cu_seqlens):
         ko.append(K[h, idx])
         vo.append(V[h, idx])
     return np.concatenate(ko, axis=0), np.concatenate(vo, axis=0)
+
+
+def decode_attention(q, K_out, V_out, cu_seqlens) -> np.ndarray:
+    """out[qh, t] = sum_i softmax_i(q[qh, t] . K_out[c + i] / sqrt(d)) V_out[c + i].
+
+    q: [Hq, n_tok, d]; K_out, V_out: [sum b_h, d] (bf16 bits or floats), the flat cache of
+    ``gather``; cu_seqlens: [Hkv + 1].  Query head qh reads the rows of KV head qh // G,
+    i in [0, cu[h+1] - cu[h]), c = cu[h].  Float64 throughout; returns float64
+    [Hq, n_tok, d]; a head without rows gives zeros.
+    """
+    qf = bf16_bits_to_f64(q) if np.asarray(q).dtype == np.uint16 else np.asarray(q, np.float64)
+    kf = bf16_bits_to_f64(K_out) if np.asarray(K_out).dtype == np.uint16 else np.asarray(K_out, np.float64)
+    vf = bf16_bits_to_f64(V_out) if np.asarray(V_out).dtype == np.uint16 else np.asarray(V_out, np.float64)
+    cu = np.asarray(cu_seqlens, dtype=np.int64)
+    Hq, n_tok, d = qf.shape
+    Hkv = cu.size - 1
+    G = Hq // Hkv
+    out = np.zeros((Hq, n_tok, d), dtype=np.float64)
+    for qh in range(Hq):
+        h = qh // G
+        rows = slice(int(cu[h]), int(cu[h + 1]))
+        if cu[h + 1] == cu[h]:
+            continue
+        logits = (qf[qh] @ kf[rows].T) / math.sqrt(d)          # [n_tok, rows]
+        m = logits.max(axis=1, keepdims=True)
+        e = np.exp(logits - m)
+        p = e / e.sum(axis=1, keepdims=True)
+        out[qh] = p @ vf[rows]
+    return out
 
 
 def compress_layer(q_win, K, V, budgets, n_sink, n_recent, pool=7, causal=True):
