@@ -46,6 +46,8 @@ def parse_args(argv=None):
     p.add_argument("--e2e-steps", type=int, default=4)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-decode", action="store_true",
+                   help="skip the decode-attention measurement over the compressed caches")
     p.add_argument("--cpu-child", action="store_true", help=argparse.SUPPRESS)
     return p.parse_args(argv)
 
@@ -407,6 +409,8 @@ def run_ours(args, world, rank, local):
     bytes_step = sum(path_bytes(wl, o["b"]) for o in outs)
     value = world * wl.L * Ls / (ms_max * 1e-3)
 
+    dec = None if args.no_decode else run_decode(args, wl, outs, dev, stream, peaks)
+
     e2e = None
     if not args.no_e2e and args.e2e_steps > 0:
         e2e = run_e2e(args, wl, layers, outs, n_sink, n_recent, dev, world)
@@ -433,6 +437,7 @@ def run_ours(args, world, rank, local):
         "hbm_path": {"achieved_gbs": bytes_step / (ms_max * 1e-3) / 1e9,
                      "peak_gbs": peaks["hbm"], "frac": bytes_step / (ms_max * 1e-3) / 1e9 / peaks["hbm"],
                      "bytes_per_step": bytes_step},
+        "decode_attention": dec,
         "gpu_launches": int(launches_timed),
         "schedule": "each step: budget allocation on the host, then one CUDA-graph launch of "
                     "the step's kernels (the scoring passes on one stream, max-pool + "
@@ -442,6 +447,53 @@ def run_ours(args, world, rank, local):
         "e2e": e2e,
     }
     return rec
+
+
+def run_decode(args, wl, outs, dev, stream, peaks):
+    """Decode attention over the compressed caches the step wrote (one new token per query
+    head, every layer): the layers' calls captured into one CUDA graph, W untimed and K
+    timed replays between CUDA events on the stream.  The caches of all layers (1.9 GB at
+    25 %) are larger than L2, so each layer's cache comes from HBM.  Bytes per layer: the
+    kept K and V rows read once, plus the queries and the fp32 outputs."""
+    import numpy as np
+    import torch
+    from paper_2609_03235_gb300 import sgdkv as sg
+    Ls = len(outs)
+    g = torch.Generator(device=dev).manual_seed(20260902)
+    qd = (torch.randn((wl.Hq, 1, wl.d), device=dev, generator=g) * 2.0).to(torch.bfloat16)
+    od = torch.empty((wl.Hq, 1, wl.d), dtype=torch.float32, device=dev)
+    rows = [int(np.sum(o["b"])) for o in outs]
+    ws = sg.make_decode_workspace(wl.Hq, wl.Hkv, 1, max(rows), dev)
+
+    def step(s):
+        for o in outs:
+            sg.sgdkv_decode_attention(qd, o["ko"], o["vo"], o["b"], od, ws, s)
+
+    step(stream)                                 # first-use setup outside the capture
+    torch.cuda.synchronize(dev)
+    graph = torch.cuda.CUDAGraph()
+    n0 = sg.sgdkv_launch_count()
+    with torch.cuda.graph(graph):
+        step(torch.cuda.current_stream(dev))
+    launches = sg.sgdkv_launch_count() - n0
+    for _ in range(max(args.warmup, 3)):
+        graph.replay()
+    torch.cuda.synchronize(dev)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = max(args.steps, 5)
+    t0.record(stream)
+    for _ in range(reps):
+        graph.replay()
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    us_layer = 1e3 * t0.elapsed_time(t1) / reps / Ls
+    byts = sum(r * wl.d * 2 * 2 for r in rows) / Ls + wl.Hq * wl.d * (2 + 4)
+    gbs = byts / (us_layer * 1e-6) / 1e9
+    return {"what": "one decode token per query head attending over each layer's compressed "
+                    "cache (sgdkv_decode_attention: partials + merge kernels)",
+            "us_per_layer": us_layer, "bytes_per_layer": byts, "achieved_gbs": gbs,
+            "peak_gbs": peaks["hbm"], "frac": gbs / peaks["hbm"], "bound": "hbm",
+            "layers": Ls, "replays": reps, "launches_per_replay": int(launches)}
 
 
 def run_e2e(args, wl, layers, outs, n_sink, n_recent, dev, world):

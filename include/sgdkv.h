@@ -296,6 +296,38 @@ SGDKV_API sgdkv_status sgdkv_pool_compact(const void* score_workspace, size_t sc
                                           size_t ws_bytes, void* stream);
 
 /*
+ * Decode attention over the compressed cache (what generation computes with it: Section
+ * 3.3, the kept tokens are each head's history; Appendix, Configuration, the cache is kept
+ * per KV head before the values are repeated for the query heads of a GQA group): for every
+ * query head qh and new token t,
+ *   out[qh][t] = sum_i softmax_i(q[qh][t] . K_cache[c + i] / sqrt(d)) V_cache[c + i],
+ * i over the b_h kept rows of KV head h = qh / G, c = b_0 + ... + b_{h-1} (the layout
+ * sgdkv_compact writes: pass the budgets it was given).  A head with b_h = 0 gives zeros.
+ *
+ * q         device bf16 [Hq][n_tok][d], 16-byte aligned; G * n_tok <= 16 (UNSUPPORTED
+ *           otherwise; G = Hq / Hkv)
+ * K_cache,
+ * V_cache   device bf16 [sum b_h][d], 16-byte aligned (may be NULL when every b_h is 0)
+ * budgets   HOST int64 [Hkv], b_h >= 0, sum < 2^31
+ * out       device fp32 [Hq][n_tok][d], 16-byte aligned
+ * workspace device, 256-byte aligned, sgdkv_decode_workspace_bytes(Hq, Hkv, n_tok, d,
+ *           sum b_h) bytes (0 there: shape unsupported); the per-warp partials.  The size
+ *           grows with sum b_h up to a bound (5.2 MB at Hkv = 4), so a workspace sized for
+ *           the largest cache serves every smaller one
+ * Arithmetic: logits with bf16 products and fp32 sums, softmax in fp32 (log2 units), the
+ * weights rounded to bf16 for the value sum, normalised by the sum of the rounded weights;
+ * the output is a convex combination of the head's value rows, within 2^-8 max|v| of the
+ * exact one.  Asynchronous on stream.  Errors: INVALID_ARG, UNSUPPORTED, WORKSPACE, CUDA.
+ */
+SGDKV_API size_t sgdkv_decode_workspace_bytes(int32_t Hq, int32_t Hkv, int32_t n_tok, int32_t d,
+                                              int64_t total_rows);
+SGDKV_API sgdkv_status sgdkv_decode_attention(const void* q, int32_t Hq, int32_t Hkv,
+                                              int32_t n_tok, int32_t d, const void* K_cache,
+                                              const void* V_cache, const int64_t* budgets,
+                                              float* out, void* workspace, size_t ws_bytes,
+                                              void* stream);
+
+/*
  * The whole per-layer step: sgdkv_score followed by sgdkv_compact on the same stream,
  * keeping the pooled scores in the workspace.  scores_out may be NULL; when given, it
  * receives the pooled scores as sgdkv_score would.  K must be device memory (the scorer
@@ -339,7 +371,8 @@ SGDKV_API const char* sgdkv_last_cuda_error_string(void);
 #define SGDKV_KERNEL_POOL 2          /* max-pool of the raw scores          */
 #define SGDKV_KERNEL_SELECT 3        /* threshold select and ordered compaction */
 #define SGDKV_KERNEL_GATHER 4        /* K/V row copy                        */
-#define SGDKV_KERNEL_KINDS 5
+#define SGDKV_KERNEL_DECODE 5        /* decode attention (partials, merge)  */
+#define SGDKV_KERNEL_KINDS 6
 SGDKV_API void sgdkv_debug_enable_kernel_timing(uint32_t kind_mask);
 SGDKV_API sgdkv_status sgdkv_debug_kernel_timing(int kind, double* total_ms, int64_t* launches);
 

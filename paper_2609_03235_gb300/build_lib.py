@@ -20,7 +20,7 @@ LIB = os.path.join(OUT, "libsgdkv.so")
 INCLUDE = os.path.join(ROOT, "include")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-CUDA_SOURCES = ["api.cu", "score_tc.cu", "select.cu", "timing.cu"]
+CUDA_SOURCES = ["api.cu", "score_tc.cu", "select.cu", "timing.cu", "decode.cu"]
 CXX_SOURCES = ["allocate.cpp"]
 
 

@@ -66,6 +66,8 @@ sgdkv_status check_workspace(void* ws, size_t ws_bytes, int32_t Hkv, int64_t L) 
   return SGDKV_OK;
 }
 
+constexpr size_t kDecodePartOffset = 256;   // decode workspace: status word, then partials
+
 sgdkv_status check_pool(int32_t pool) {
   if (pool < 1 || pool > 63 || pool % 2 == 0) return SGDKV_ERR_INVALID_ARG;
   return SGDKV_OK;
@@ -408,6 +410,41 @@ sgdkv_status sgdkv_compress_layer(const void* q_win, const void* K, const void* 
                                      indices_out, cu_seqlens_out,
                                      static_cast<__nv_bfloat16*>(K_out),
                                      static_cast<__nv_bfloat16*>(V_out), ws, st));
+}
+
+size_t sgdkv_decode_workspace_bytes(int32_t Hq, int32_t Hkv, int32_t n_tok, int32_t d,
+                                    int64_t total_rows) {
+  if (Hq <= 0 || Hkv <= 0 || n_tok <= 0 || d != kD || total_rows < 0) return 0;
+  if (Hq % Hkv != 0 || Hkv > SGDKV_MAX_KV_HEADS || (Hq / Hkv) * n_tok > 16) return 0;
+  if (total_rows >= (int64_t(1) << 31)) return 0;
+  return kDecodePartOffset + decode_partial_bytes(total_rows, Hkv);
+}
+
+sgdkv_status sgdkv_decode_attention(const void* q, int32_t Hq, int32_t Hkv, int32_t n_tok,
+                                    int32_t d, const void* K_cache, const void* V_cache,
+                                    const int64_t* budgets, float* out, void* workspace,
+                                    size_t ws_bytes, void* stream) {
+  if (!q || !budgets || !out) return SGDKV_ERR_INVALID_ARG;
+  if (Hq <= 0 || Hkv <= 0 || n_tok <= 0 || d <= 0 || Hq % Hkv != 0) return SGDKV_ERR_INVALID_ARG;
+  if (d != kD || Hkv > SGDKV_MAX_KV_HEADS || (Hq / Hkv) * n_tok > 16) return SGDKV_ERR_UNSUPPORTED;
+  int64_t total = 0;
+  for (int h = 0; h < Hkv; ++h) {
+    if (budgets[h] < 0) return SGDKV_ERR_INVALID_ARG;
+    total += budgets[h];
+    if (total >= (int64_t(1) << 31)) return SGDKV_ERR_UNSUPPORTED;
+  }
+  if (total > 0 && (!K_cache || !V_cache)) return SGDKV_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(out) || (total > 0 && (!aligned16(K_cache) || !aligned16(V_cache))))
+    return SGDKV_ERR_INVALID_ARG;
+  const size_t need = sgdkv_decode_workspace_bytes(Hq, Hkv, n_tok, d, total);
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0 || ws_bytes < need)
+    return SGDKV_ERR_WORKSPACE;
+  float* part = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) + kDecodePartOffset);
+  return from_cuda(launch_decode(static_cast<const __nv_bfloat16*>(q),
+                                 static_cast<const __nv_bfloat16*>(K_cache),
+                                 static_cast<const __nv_bfloat16*>(V_cache), budgets, Hq, Hkv,
+                                 n_tok, out, part, ws_bytes - kDecodePartOffset,
+                                 static_cast<cudaStream_t>(stream)));
 }
 
 sgdkv_status sgdkv_last_error(void* workspace, void* stream) {

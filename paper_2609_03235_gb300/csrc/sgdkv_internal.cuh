@@ -117,4 +117,13 @@ cudaError_t launch_compact(const __nv_bfloat16* K, const __nv_bfloat16* V,
 // can take a PoolSrc
 bool compact_pools_inline(int64_t L);
 
+// Decode attention over the flat compressed cache (decode.cu): bytes of the per-warp
+// partials for total_rows kept rows, and the launcher (q [Hq][T][128], K/V cache
+// [sum b_h][128], out fp32 [Hq][T][128]; budgets on the host).
+size_t decode_partial_bytes(int64_t total_rows, int Hkv);
+cudaError_t launch_decode(const __nv_bfloat16* q, const __nv_bfloat16* Kc,
+                          const __nv_bfloat16* Vc, const int64_t* budgets, int Hq, int Hkv,
+                          int T, float* out, float* part, size_t part_bytes,
+                          cudaStream_t stream);
+
 }  // namespace sgdkv

@@ -23,7 +23,8 @@ EXPORTED = ("sgdkv_status_string", "sgdkv_version", "sgdkv_allocate_budgets",
             "sgdkv_last_cuda_error_string", "sgdkv_score_static",
             "sgdkv_debug_enable_kernel_timing", "sgdkv_debug_kernel_timing", "sgdkv_score_ex",
             "sgdkv_mix_head_scores", "sgdkv_score_raw", "sgdkv_pool_raw",
-            "sgdkv_window_stats", "sgdkv_window_sums", "sgdkv_pool_compact")
+            "sgdkv_window_stats", "sgdkv_window_sums", "sgdkv_pool_compact",
+            "sgdkv_decode_workspace_bytes", "sgdkv_decode_attention")
 
 
 class LibraryMissing(RuntimeError):
@@ -83,6 +84,11 @@ def lib():
             fn.argtypes = [_P, _P, _I32, _I32, _I64, _I32, _I32, ctypes.c_uint32, _P, _P, _SZ, _P]
         L.sgdkv_pool_raw.restype = ctypes.c_int
         L.sgdkv_pool_raw.argtypes = [_P, _SZ, _I32, _I64, _I32, ctypes.c_uint32, _P, _P]
+        L.sgdkv_decode_workspace_bytes.restype = _SZ
+        L.sgdkv_decode_workspace_bytes.argtypes = [_I32, _I32, _I32, _I32, _I64]
+        L.sgdkv_decode_attention.restype = ctypes.c_int
+        L.sgdkv_decode_attention.argtypes = [_P, _I32, _I32, _I32, _I32, _P, _P, _P, _P, _P,
+                                             _SZ, _P]
         L.sgdkv_pool_compact.restype = ctypes.c_int
         L.sgdkv_pool_compact.argtypes = [_P, _SZ, _I32, ctypes.c_uint32, _P, _P, _P, _I32, _I64,
                                          _I32, _I64, _I64, _P, _P, _P, _P, _P, _P, _SZ, _P]
@@ -260,6 +266,31 @@ def sgdkv_pool_compact(score_workspace, pool: int, K, V, budgets, n_sink: int, n
     _check(st, "sgdkv_pool_compact")
 
 
+def sgdkv_decode_workspace_bytes(Hq: int, Hkv: int, n_tok: int, d: int, total_rows: int) -> int:
+    return int(lib().sgdkv_decode_workspace_bytes(int(Hq), int(Hkv), int(n_tok), int(d),
+                                                  int(total_rows)))
+
+
+def make_decode_workspace(Hq: int, Hkv: int, n_tok: int, total_rows: int, device="cuda",
+                          d: int = 128):
+    """Workspace tensor for sgdkv_decode_attention (caller-owned device memory)."""
+    import torch
+    n = sgdkv_decode_workspace_bytes(Hq, Hkv, n_tok, d, total_rows)
+    if n == 0:
+        raise SgdkvError(ERR_UNSUPPORTED, "sgdkv_decode_workspace_bytes")
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def sgdkv_decode_attention(q, K_cache, V_cache, budgets, out, workspace, stream=None):
+    """Attention of q [Hq][n_tok][d] over the compressed cache; out fp32 [Hq][n_tok][d]."""
+    Hq, n_tok, d = q.shape
+    b = _budgets(budgets)
+    st = lib().sgdkv_decode_attention(_ptr(q), Hq, len(b), n_tok, d, _ptr(K_cache),
+                                      _ptr(V_cache), b.ctypes.data_as(_P), _ptr(out),
+                                      _ptr(workspace), workspace.numel(), _stream(stream))
+    _check(st, "sgdkv_decode_attention")
+
+
 def sgdkv_compress_layer(q_win, K, V, budgets, W: int, pool: int, n_sink: int, n_recent: int,
                          scores_out, indices_out, cu_seqlens_out, K_out, V_out, workspace,
                          stream=None):
@@ -282,7 +313,8 @@ def sgdkv_debug_set_score_hooks(flags: int, wait_ns: int = 0) -> None:
     lib().sgdkv_debug_set_score_hooks(int(flags), int(wait_ns))
 
 
-KERNEL_SCORE_PASS1, KERNEL_SCORE_PASS2, KERNEL_POOL, KERNEL_SELECT, KERNEL_GATHER = range(5)
+KERNEL_SCORE_PASS1, KERNEL_SCORE_PASS2, KERNEL_POOL, KERNEL_SELECT, KERNEL_GATHER, \
+    KERNEL_DECODE = range(6)
 
 
 def sgdkv_debug_enable_kernel_timing(kinds=()) -> None:

@@ -200,6 +200,35 @@ def test_score_rejects_bad_args_before_device_work():
     assert call(ws=16) == sg.ERR_WORKSPACE                    # compaction workspace too small
 
 
+def test_decode_rejects_bad_args_before_device_work():
+    import ctypes
+    L = sg.lib()
+    wb = L.sgdkv_decode_workspace_bytes
+    assert wb(28, 4, 1, 128, 131072) > 0
+    assert wb(28, 4, 1, 128, 0) > 0
+    assert wb(28, 4, 1, 64, 1000) == 0             # head dim
+    assert wb(28, 4, 3, 128, 1000) == 0            # G * n_tok = 21 > 16
+    assert wb(28, 5, 1, 128, 1000) == 0            # Hq % Hkv
+    assert wb(28, 4, 1, 128, -1) == 0
+    buf = (ctypes.c_uint8 * 4096)()
+    p = ctypes.cast(buf, ctypes.c_void_p)
+    good = np.array([100, 200, 0, 50], np.int64)
+    neg = np.array([100, -1, 0, 50], np.int64)
+    da = L.sgdkv_decode_attention
+
+    def call(q=p, Hq=28, n_tok=1, d=128, b=good, out=p, ws_bytes=1 << 30):
+        return da(q, Hq, 4, n_tok, d, p, p, b.ctypes.data_as(ctypes.c_void_p), out, p,
+                  ws_bytes, None)
+    assert call(q=None) == sg.ERR_INVALID_ARG
+    assert call(out=None) == sg.ERR_INVALID_ARG
+    assert call(d=64) == sg.ERR_UNSUPPORTED
+    assert call(n_tok=3) == sg.ERR_UNSUPPORTED
+    assert call(Hq=30) == sg.ERR_INVALID_ARG
+    assert call(b=neg) == sg.ERR_INVALID_ARG
+    assert call(ws_bytes=16) == sg.ERR_WORKSPACE
+    assert da(p, 28, 4, 1, 128, p, p, None, p, p, 1 << 30, None) == sg.ERR_INVALID_ARG
+
+
 def test_compact_rejects_bad_budgets():
     import ctypes
     L = sg.lib()
