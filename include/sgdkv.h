@@ -312,7 +312,7 @@ SGDKV_API sgdkv_status sgdkv_pool_compact(const void* score_workspace, size_t sc
  * out       device fp32 [Hq][n_tok][d], 16-byte aligned
  * workspace device, 256-byte aligned, sgdkv_decode_workspace_bytes(Hq, Hkv, n_tok, d,
  *           sum b_h) bytes (0 there: shape unsupported); the per-warp partials.  The size
- *           grows with sum b_h up to a bound (5.2 MB at Hkv = 4), so a workspace sized for
+ *           grows with sum b_h up to a bound (1.3 MB at Hkv = 4), so a workspace sized for
  *           the largest cache serves every smaller one
  * Arithmetic: logits with bf16 products and fp32 sums, softmax in fp32 (log2 units), the
  * weights rounded to bf16 for the value sum, normalised by the sum of the rounded weights;

@@ -7,34 +7,36 @@
 //
 // The work is a stream of the kept K and V rows (HBM-bound: G * T <= 16 query rows meet
 // every K row once and every V row once).  Each warp takes a contiguous chunk of one head's
-// rows and streams it through a three-stage ring of 32-row K and V tiles in its own shared
+// rows (a quarter of its CTA's chunk) and streams it through a three-stage ring of 32-row K
+// and V tiles in its own shared
 // memory (cp.async, 16-byte chunks, XOR-swizzled so that the matrix loads are free of bank
 // conflicts).  Per tile, 16 x 32 logits come from mma.m16n8k16 (bf16, fp32 accumulate; the
 // query rows of the group are the 16 rows of A, padded with zeros), an online softmax in
 // log2 units runs per query row across the four threads that hold it, and the weights,
 // rounded to bf16, multiply the V tile in a second mma chain into 16 x 128 fp32
 // accumulators.  The row sums are taken over the rounded weights, so every output is a
-// convex combination of the head's value rows.  Each warp leaves (max, sum, 128 sums) per
-// query row; a second kernel merges a head's partials.
+// convex combination of the head's value rows.  The four warps of a CTA merge their (max,
+// sum, 128 sums) per query row in shared memory into one partial per CTA chunk; a second
+// kernel merges a head's partials.
 #include "sgdkv_internal.cuh"
 
 namespace sgdkv {
 namespace {
 
-constexpr int kDWarps = 4;                 // warps per CTA (independent chunks)
+constexpr int kDWarps = 4;                 // warps per CTA (a quarter of the CTA's chunk each)
 constexpr int kDTile = 32;                 // rows per tile
 constexpr int kDStages = 3;                // tiles in flight per warp
 constexpr int kDTileBytes = kDTile * kD * 2;            // 8 KB of K or of V
 constexpr int kDWarpBytes = kDStages * 2 * kDTileBytes;  // 48 KB per warp
 constexpr int kDPartStride = kD + 4;       // floats per partial row: 128 sums, max, sum, pad
-constexpr int kDTargetWarps = 152 * kDWarps;   // warp chunks per call: one wave on 152 SMs
+constexpr int kDTargetChunks = 152;       // CTA chunks per call: one wave on 152 SMs
 
 struct DecodeParams {
   int Hkv, G, T, nq;                       // nq = G * T query rows per head (<= 16)
-  int chunk;                               // rows per warp chunk (a multiple of kDTile)
+  int chunk;                               // rows per CTA chunk (a multiple of kDWarps*kDTile)
   float scale2;                            // log2(e) / sqrt(d)
   int32_t cu[SGDKV_MAX_KV_HEADS + 1];      // first row of each head in the flat cache
-  int32_t wpfx[SGDKV_MAX_KV_HEADS + 1];    // first warp chunk of each head
+  int32_t wpfx[SGDKV_MAX_KV_HEADS + 1];    // first CTA chunk of each head
 };
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
@@ -97,12 +99,14 @@ decode_partial_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* 
   extern __shared__ __align__(128) uint8_t dsm[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, t = lane & 3;
-  const int wg = blockIdx.x * kDWarps + warp;            // global warp chunk
-  if (wg >= p.wpfx[p.Hkv]) return;
+  const int cg = blockIdx.x;                             // CTA chunk (grid = chunks)
   int h = 0;
-  while (wg >= p.wpfx[h + 1]) ++h;
-  const int row0 = p.cu[h] + (wg - p.wpfx[h]) * p.chunk;
-  const int row_end = min(row0 + p.chunk, p.cu[h + 1]);
+  while (cg >= p.wpfx[h + 1]) ++h;
+  const int c0 = p.cu[h] + (cg - p.wpfx[h]) * p.chunk;
+  const int c1 = min(c0 + p.chunk, p.cu[h + 1]);
+  const int sub = p.chunk / kDWarps;                     // this warp: a quarter of the chunk
+  const int row0 = min(c0 + warp * sub, c1);
+  const int row_end = min(row0 + sub, c1);
   const int ntiles = (row_end - row0 + kDTile - 1) / kDTile;
   uint8_t* wbase = dsm + warp * kDWarpBytes;
   const uint32_t sbase = smem_addr(wbase);
@@ -232,18 +236,43 @@ decode_partial_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* 
   l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
   l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
   l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-  float* pr0 = part + (size_t(wg) * 16 + g) * kDPartStride;
-  float* pr1 = part + (size_t(wg) * 16 + g + 8) * kDPartStride;
+  // the four warps' (max, sum, 128 sums) per row, in the rings' shared memory once every
+  // warp is done with its ring, merged by one thread per column into the CTA's partial
+  __syncthreads();
+  float* red = reinterpret_cast<float*>(dsm);            // [kDWarps][16][kDPartStride]
+  float* r0 = red + (warp * 16 + g) * kDPartStride;
+  float* r1 = red + (warp * 16 + g + 8) * kDPartStride;
 #pragma unroll
   for (int n = 0; n < 16; ++n) {
-    *reinterpret_cast<float2*>(pr0 + 8 * n + 2 * t) = make_float2(o[n][0], o[n][1]);
-    *reinterpret_cast<float2*>(pr1 + 8 * n + 2 * t) = make_float2(o[n][2], o[n][3]);
+    *reinterpret_cast<float2*>(r0 + 8 * n + 2 * t) = make_float2(o[n][0], o[n][1]);
+    *reinterpret_cast<float2*>(r1 + 8 * n + 2 * t) = make_float2(o[n][2], o[n][3]);
   }
   if (t == 0) {
-    pr0[kD] = m0;
-    pr0[kD + 1] = l0;
-    pr1[kD] = m1;
-    pr1[kD + 1] = l1;
+    r0[kD] = m0;
+    r0[kD + 1] = l0;
+    r1[kD] = m1;
+    r1[kD + 1] = l1;
+  }
+  __syncthreads();
+  const int d = threadIdx.x;                             // kDWarps * 32 == kD columns
+  for (int r = 0; r < p.nq; ++r) {
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < kDWarps; ++w) M = fmaxf(M, red[(w * 16 + r) * kDPartStride + kD]);
+    float S = 0.f, O = 0.f;
+#pragma unroll
+    for (int w = 0; w < kDWarps; ++w) {
+      const float* rw = red + (w * 16 + r) * kDPartStride;
+      const float f = rw[kD] == -INFINITY ? 0.f : ex2f(rw[kD] - M);
+      S += f * rw[kD + 1];
+      O += f * rw[d];
+    }
+    float* pr = part + (size_t(cg) * 16 + r) * kDPartStride;
+    pr[d] = O;
+    if (d == 0) {
+      pr[kD] = M;
+      pr[kD + 1] = S;
+    }
   }
 }
 
@@ -252,7 +281,7 @@ decode_partial_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* 
 // partial max and the weights 2^(m_w - M) with their normaliser are formed once in shared
 // memory, then four groups of 128 threads (one per column) sum interleaved partials.
 constexpr int kDCombThreads = 512;
-constexpr int kDMaxChunks = 1024;              // > kDTargetWarps + SGDKV_MAX_KV_HEADS
+constexpr int kDMaxChunks = 1024;              // >= kDTargetChunks + SGDKV_MAX_KV_HEADS
 
 __device__ __forceinline__ float block_reduce(float v, bool is_max, float* red) {
 #pragma unroll
@@ -312,20 +341,23 @@ decode_combine_kernel(const float* __restrict__ part, DecodeParams p, float* __r
 
 }  // namespace
 
-// Rows per warp chunk: about kDTargetWarps chunks per call, in whole tiles (a function of
-// the total rows alone, so that the workspace size does not depend on the device).
+// Rows per CTA chunk: about kDTargetChunks chunks per call, a whole tile per warp (a
+// function of the total rows alone, so that the workspace size does not depend on the
+// device).
 int decode_chunk_rows(int64_t total_rows) {
-  int64_t c = ceil_div(total_rows > 0 ? total_rows : 1, kDTargetWarps);
-  c = ceil_div(c, kDTile) * kDTile;
+  constexpr int kQuant = kDWarps * kDTile;
+  int64_t c = ceil_div(total_rows > 0 ? total_rows : 1, kDTargetChunks);
+  c = ceil_div(c, kQuant) * kQuant;
   return int(c);
 }
 
-// Bytes of the partials: one per warp chunk, at most min(ceil(rows / kDTile), kDTargetWarps)
-// + Hkv of them (a chunk holds >= kDTile and >= rows / kDTargetWarps rows).  The bound grows
-// with total_rows, so a workspace sized for the largest cache serves every smaller one.
+// Bytes of the partials: one per CTA chunk, at most min(ceil(rows / (kDWarps * kDTile)),
+// kDTargetChunks) + Hkv of them (a chunk holds >= kDWarps * kDTile and >= rows /
+// kDTargetChunks rows).  The bound grows with total_rows, so a workspace sized for the
+// largest cache serves every smaller one.
 size_t decode_partial_bytes(int64_t total_rows, int Hkv) {
-  int64_t n = ceil_div(total_rows, kDTile);
-  if (n > kDTargetWarps) n = kDTargetWarps;
+  int64_t n = ceil_div(total_rows, kDWarps * kDTile);
+  if (n > kDTargetChunks) n = kDTargetChunks;
   return size_t(n + Hkv) * 16 * kDPartStride * sizeof(float);
 }
 
@@ -348,16 +380,18 @@ cudaError_t launch_decode(const __nv_bfloat16* q, const __nv_bfloat16* Kc,
     p.cu[h + 1] = p.cu[h] + int32_t(budgets[h]);
     p.wpfx[h + 1] = p.wpfx[h] + int32_t(ceil_div(budgets[h], p.chunk));
   }
-  const int nwarps = p.wpfx[Hkv];
-  static_assert(kDMaxChunks >= kDTargetWarps + SGDKV_MAX_KV_HEADS, "chunks per head");
-  if (size_t(nwarps) * 16 * kDPartStride * sizeof(float) > part_bytes) return cudaErrorInvalidValue;
+  const int nchunks = p.wpfx[Hkv];
+  static_assert(kDMaxChunks >= kDTargetChunks + SGDKV_MAX_KV_HEADS, "chunks per head");
+  static_assert(kDWarps * 32 == kD, "one merge thread per column");
+  static_assert(kDWarps * 16 * kDPartStride * 4 <= kDWarps * kDWarpBytes, "merge buffer");
+  if (size_t(nchunks) * 16 * kDPartStride * sizeof(float) > part_bytes) return cudaErrorInvalidValue;
   const int smem = kDWarps * kDWarpBytes;
   cudaError_t e = cudaFuncSetAttribute(decode_partial_kernel,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  if (nwarps > 0) {
+  if (nchunks > 0) {
     KernelTimer tk(SGDKV_KERNEL_DECODE, stream);
-    decode_partial_kernel<<<unsigned(ceil_div(nwarps, kDWarps)), kDWarps * 32, smem, stream>>>(
+    decode_partial_kernel<<<unsigned(nchunks), kDWarps * 32, smem, stream>>>(
         q, Kc, Vc, p, part);
     note_launches(1);
   }
