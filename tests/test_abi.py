@@ -229,6 +229,19 @@ def test_decode_rejects_bad_args_before_device_work():
     assert da(p, 28, 4, 1, 128, p, p, None, p, p, 1 << 30, None) == sg.ERR_INVALID_ARG
 
 
+def test_decode_workspace_bound_grows_with_the_cache():
+    """A decode workspace sized for the largest cache serves every smaller one: the size is
+    non-decreasing in the total kept rows and stops growing at its bound."""
+    prev = 0
+    for rows in list(range(0, 40000, 61)) + [131072, 524288, 2 ** 31 - 1]:
+        n = sg.sgdkv_decode_workspace_bytes(28, 4, 1, 128, rows)
+        assert n >= prev > 0 or (prev == 0 and n > 0)
+        prev = n
+    assert sg.sgdkv_decode_workspace_bytes(28, 4, 1, 128, 2 ** 31 - 1) == \
+        sg.sgdkv_decode_workspace_bytes(28, 4, 1, 128, 10 ** 9)
+    assert sg.sgdkv_decode_workspace_bytes(28, 4, 1, 128, 2 ** 31) == 0
+
+
 def test_compact_rejects_bad_budgets():
     import ctypes
     L = sg.lib()
