@@ -46,6 +46,8 @@ def parse_args(argv=None):
     p.add_argument("--e2e-steps", type=int, default=4)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-sweep", action="store_true",
+                   help="skip the per-workload measurements beside the headline")
     p.add_argument("--no-decode", action="store_true",
                    help="skip the decode-attention measurement over the compressed caches")
     p.add_argument("--cpu-child", action="store_true", help=argparse.SUPPRESS)
@@ -251,200 +253,302 @@ def workload_config(wl, args, world, n_layers):
 
 
 
-def run_ours(args, world, rank, local):
-    import numpy as np
+class StepRunner:
+    """One workload's compression step on this GPU: inputs of every layer resident in HBM,
+    the step's launches captured into CUDA graphs and replayed.
+
+    One step = the host budget allocation (a1), then the launches of every layer: the two
+    scoring passes on the capturing stream, sgdkv_pool_compact (the max-pool inside the
+    selection kernel, then the gather) on `sel_stream`; layer l's pooling and compaction
+    wait for layer l's passes only, so they overlap layer l+1's scoring, whose CTAs claim
+    key tiles dynamically and absorb the SMs the other stream leaves.  The raw scores of
+    layer l stay in scoring workspace l % 3 until its compaction has read them (layer
+    l + 3's scoring waits for that: with two workspaces, layer l + 2's scoring would wait
+    for layer l's gather as well).  The launches of a step are captured into a CUDA graph
+    (per-kernel launch cost ~1 us instead of ~3 us on a stream) and the graph is replayed;
+    the allocation still runs on the host every step and must reproduce the budgets the
+    graph was captured with."""
+
+    def __init__(self, wl, frac, n_layers, dev):
+        import numpy as np
+        import torch
+
+        from paper_2609_03235_gb300 import configs, synth
+        from paper_2609_03235_gb300 import sgdkv as sg
+        self.np, self.torch, self.sg = np, torch, sg
+        self.wl, self.frac, self.dev = wl, frac, dev
+        self.n_sink, self.n_recent = configs.sink_recent_split(wl.floor)
+        self.hs = synth.head_scores(wl)
+        self.T = wl.total_budget(frac)
+        self.b_all = sg.sgdkv_allocate_budgets(self.hs, wl.L, self.T, wl.floor)
+        self.Ls = n_layers
+        self.layers = [synth.layer_inputs_device(wl, l, dev) for l in range(n_layers)]
+        self.outs = []
+        for l in range(n_layers):
+            b = self.b_all[l * wl.Hkv:(l + 1) * wl.Hkv]
+            tot = int(b.sum())
+            self.outs.append(dict(
+                b=b, scores=torch.empty((wl.Hkv, wl.L), dtype=torch.float32, device=dev),
+                idx=torch.empty(tot, dtype=torch.int32, device=dev),
+                cu=torch.empty(wl.Hkv + 1, dtype=torch.int32, device=dev),
+                ko=torch.empty((tot, wl.d), dtype=torch.bfloat16, device=dev),
+                vo=torch.empty((tot, wl.d), dtype=torch.bfloat16, device=dev)))
+        self.ws_score = [sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
+                         for _ in range(N_SCORE_WS)]
+        self.ws_sel = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
+        self.stream = torch.cuda.current_stream(dev)
+        lo_prio, hi_prio = torch.cuda.Stream.priority_range()
+        self.sel_stream = torch.cuda.Stream(dev, priority=hi_prio)
+        self.fork = torch.cuda.Event()
+        self.scored = [torch.cuda.Event() for _ in range(n_layers)]
+        self.pooled = [torch.cuda.Event() for _ in range(n_layers)]  # workspace l % N read
+        self.done = torch.cuda.Event()
+
+    def launches(self, s, kinds=(), every=1, first=0):
+        sg, wl = self.sg, self.wl
+        self.fork.record(s)
+        self.sel_stream.wait_event(self.fork)
+        for l in range(self.Ls):
+            inp, o = self.layers[l], self.outs[l]
+            sg.sgdkv_debug_enable_kernel_timing(kinds if l % every == first % every else ())
+            wsl = self.ws_score[l % N_SCORE_WS]
+            if l >= N_SCORE_WS:
+                s.wait_event(self.pooled[l - N_SCORE_WS])   # its workspace read by then
+            sg.sgdkv_score_raw(inp["q"], inp["K"], wl.W, wsl, s)
+            self.scored[l].record(s)
+            self.sel_stream.wait_event(self.scored[l])
+            sg.sgdkv_pool_compact(wsl, wl.pool, inp["K"], inp["V"], o["b"], self.n_sink,
+                                  self.n_recent, o["scores"], o["idx"], o["cu"], o["ko"],
+                                  o["vo"], self.ws_sel, self.sel_stream)
+            self.pooled[l].record(self.sel_stream)
+        sg.sgdkv_debug_enable_kernel_timing(())
+        self.done.record(self.sel_stream)
+        s.wait_event(self.done)
+
+    def allocate(self):
+        ball = self.sg.sgdkv_allocate_budgets(self.hs, self.wl.L, self.T, self.wl.floor)   # a1
+        if not self.np.array_equal(ball, self.b_all):
+            raise RuntimeError("budget allocation changed between steps")
+        return ball
+
+    def capture(self, kinds, every=1, first=0):
+        """One step's launches as a CUDA graph; the kernels of `kinds` in every `every`-th
+        layer from layer `first` on are bracketed by timing events."""
+        torch, sg = self.torch, self.sg
+        g = torch.cuda.CUDAGraph()
+        n0 = sg.sgdkv_launch_count()
+        with torch.cuda.graph(g):
+            self.launches(torch.cuda.current_stream(self.dev), kinds, every, first)
+        return g, sg.sgdkv_launch_count() - n0
+
+    def drain_timers(self):
+        return [self.sg.sgdkv_debug_kernel_timing(kind) for kind in range(len(KERNEL_NAMES))]
+
+    def check(self, where):
+        sg = self.sg
+        st = max(max(sg.sgdkv_last_error(w, self.stream) for w in self.ws_score),
+                 sg.sgdkv_last_error(self.ws_sel, self.sel_stream))
+        if st != sg.OK:
+            raise RuntimeError(f"device-side error {where}: {sg.status_string(st)}")
+
+    def measure(self, steps, warmup, diag_steps, world, local):
+        """Warm-up, a diagnostic window (every launch bracketed: per-kernel shares and the
+        dominant scoring pass), then `steps` timed graph replays between barrier +
+        synchronize and CUDA events on the launching stream, with the dominant pass
+        bracketed in every TIMED_EVERY-th layer (rotating by one layer per step) and
+        nvidia-smi clocks sampled meanwhile."""
+        torch = self.torch
+        dev = self.dev
+        self.launches(self.stream)         # one eager step (first-use setup), then graphs
+        torch.cuda.synchronize(dev)
+        self.check("in the first step")
+        g_warm, _ = self.capture(())
+        for _ in range(max(warmup, 0)):
+            self.allocate()
+            g_warm.replay()
+        torch.cuda.synchronize(dev)
+        self.check("during warm-up")
+        self.drain_timers()
+        diag = [self.capture(range(len(KERNEL_NAMES)))[0] for _ in range(diag_steps)]
+        for g in diag:
+            self.allocate()
+            g.replay()
+        torch.cuda.synchronize(dev)
+        kern = {}
+        for name, (tot_ms, n) in zip(KERNEL_NAMES, self.drain_timers()):
+            kern[name] = {"launches": n, "us_per_launch": 1e3 * tot_ms / max(n, 1),
+                          "ms_total": tot_ms, "dram_bytes_ncu": measured_traffic(name, self.wl.name)}
+        del diag
+        kern = {k: v for k, v in kern.items() if v["launches"] > 0}
+        all_ms = sum(v["ms_total"] for v in kern.values())
+        for v in kern.values():
+            v["share"] = v["ms_total"] / all_ms if all_ms > 0 else None
+        top_kind = max(range(2), key=lambda k: kern[KERNEL_NAMES[k]]["ms_total"])
+        timed = [self.capture([top_kind], TIMED_EVERY, k) for k in range(steps)]
+        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        clocks = ClockSampler(nvsmi_id(local))
+        barrier(world)
+        torch.cuda.synchronize(dev)
+        clocks.start()
+        time.sleep(0.3)                  # let the sampler attach before the timed region
+        start.record(self.stream)
+        for g, _ in timed:
+            self.allocate()
+            g.replay()
+        end.record(self.stream)
+        torch.cuda.synchronize(dev)
+        launches_timed = sum(n for _, n in timed)
+        top_ms, top_n = self.sg.sgdkv_debug_kernel_timing(top_kind)
+        clk = clocks.stop()
+        barrier(world)
+        self.check("in the timed region")
+        del timed, g_warm
+        ms = start.elapsed_time(end) / steps
+        return dict(ms=ms, ms_max=max_over_ranks(ms, world), kern=kern,
+                    top=KERNEL_NAMES[top_kind], top_us=1e3 * top_ms / max(top_n, 1),
+                    top_n=top_n, launches=int(launches_timed), clocks=clk)
+
+    def free(self):
+        self.layers = self.outs = self.ws_score = self.ws_sel = None
+
+
+def roofs(wl, outs, ms_step, n_layers, peaks):
+    """The step against its two roofs (per layer): HBM for the algorithmic bytes and the
+    tensor pipe for the two scoring passes' flops.  The binding roof is the larger of the two
+    floor times; its fraction is floor time / measured time."""
+    bytes_step = sum(path_bytes(wl, o["b"]) for o in outs)
+    us_layer = 1e3 * ms_step / n_layers
+    hbm_us = bytes_step / n_layers / (peaks["hbm"] * 1e9) * 1e6
+    tensor_us = score_flops(wl) / (peaks["bf16"] * 1e12) * 1e6
+    bound = "tensor" if tensor_us > hbm_us else "hbm"
+    roof_us = max(hbm_us, tensor_us)
+    hbm_gbs = bytes_step / (ms_step * 1e-3) / 1e9
+    return bytes_step, {
+        "hbm_path": {"achieved_gbs": hbm_gbs, "peak_gbs": peaks["hbm"],
+                     "frac": hbm_gbs / peaks["hbm"], "bytes_per_step": bytes_step},
+        "binding_roof": {"bound": bound, "floor_us_per_layer": roof_us,
+                         "hbm_floor_us_per_layer": hbm_us, "tensor_floor_us_per_layer": tensor_us,
+                         "us_per_layer": us_layer, "frac": roof_us / us_layer,
+                         "peaks": f"{peaks['source']}: HBM {peaks['hbm']} GB/s, bf16 burst "
+                                  f"{peaks['bf16']} TFLOP/s (two scoring passes of "
+                                  "2*G*W*d flops per key per KV head)"}}
+
+
+# Workloads measured beside the headline by the default run: every configuration the
+# compression step is specified on, the 128K Qwen2.5-7B shape at each of its total budgets.
+SWEEP_STEPS, SWEEP_WARMUP = 5, 3
+
+
+def sweep_cases():
+    from paper_2609_03235_gb300 import configs
+    return [(w.name, f) for w in configs.WORKLOADS for f in w.budget_fracs]
+
+
+def run_sweep(args, world, local, dev, peaks, skip):
+    """One entry per (workload, total budget): tokens/s/layer, us/layer, the HBM and binding
+    roof fractions, the dominant pass's CUDA-event time and the clocks of its timed region."""
     import torch
 
-    from paper_2609_03235_gb300 import configs, synth
+    from paper_2609_03235_gb300 import configs
+    out = {}
+    for name, frac in sweep_cases():
+        key = f"{name}@{frac:g}"
+        if (name, frac) == skip:
+            out[key] = "headline (top-level fields of this line)"
+            continue
+        wl = configs.BY_NAME[name]
+        r = StepRunner(wl, frac, wl.n_layers, dev)
+        m = r.measure(SWEEP_STEPS, SWEEP_WARMUP, 1, world, local)
+        _, rf = roofs(wl, r.outs, m["ms_max"], r.Ls, peaks)
+        tf = pass_flops(wl) / (m["top_us"] * 1e-6) / 1e12
+        out[key] = {
+            "value": world * wl.L * r.Ls / (m["ms_max"] * 1e-3), "unit": UNIT,
+            "us_per_layer": 1e3 * m["ms_max"] / r.Ls, "ms_per_step": m["ms_max"],
+            "n_layers": r.Ls, "steps": SWEEP_STEPS, "warmup": SWEEP_WARMUP,
+            "model_shape": "Qwen2.5-7B-1M" if wl.Hkv == 4 else "Qwen3-32B",
+            "context_len": wl.L, "window": wl.W, "budget_frac": frac,
+            **rf,
+            "dominant_pass": {"kernel": m["top"], "us_per_launch": m["top_us"],
+                              "launches_timed": m["top_n"], "tflops": tf,
+                              "frac_of_bf16_burst": tf / peaks["bf16"]},
+            "gpu_launches": m["launches"], "clocks": m["clocks"]}
+        r.free()
+        del r
+        torch.cuda.synchronize(dev)
+        torch.cuda.empty_cache()
+    return out
+
+
+def run_ours(args, world, rank, local):
+    import torch
+
+    from paper_2609_03235_gb300 import configs
     from paper_2609_03235_gb300 import sgdkv as sg
 
     wl = configs.BY_NAME[args.workload]
     dev = torch.device(f"cuda:{local}")
     torch.cuda.set_device(dev)
     sg.lib()
-    n_sink, n_recent = configs.sink_recent_split(wl.floor)
-    hs = synth.head_scores(wl)
-    T = wl.total_budget(args.frac)
-    b_all = sg.sgdkv_allocate_budgets(hs, wl.L, T, wl.floor)
     Ls = wl.n_layers if args.layers <= 0 else min(args.layers, wl.n_layers)
-    layers = [synth.layer_inputs_device(wl, l, dev) for l in range(Ls)]
-    outs = []
-    for l in range(Ls):
-        b = b_all[l * wl.Hkv:(l + 1) * wl.Hkv]
-        tot = int(b.sum())
-        outs.append(dict(
-            b=b, scores=torch.empty((wl.Hkv, wl.L), dtype=torch.float32, device=dev),
-            idx=torch.empty(tot, dtype=torch.int32, device=dev),
-            cu=torch.empty(wl.Hkv + 1, dtype=torch.int32, device=dev),
-            ko=torch.empty((tot, wl.d), dtype=torch.bfloat16, device=dev),
-            vo=torch.empty((tot, wl.d), dtype=torch.bfloat16, device=dev)))
-    # One step = the host budget allocation (a1), then the launches of every layer: the two
-    # scoring passes on the capturing stream, sgdkv_pool_compact (the max-pool inside the
-    # selection kernel, then the gather) on `sel_stream`; layer l's pooling and compaction
-    # wait for layer l's passes only, so they overlap layer l+1's scoring, whose CTAs claim
-    # key tiles dynamically and absorb the SMs the other stream leaves.  The raw scores of
-    # layer l stay in scoring workspace l % 3 until its compaction has read them (layer
-    # l + 3's scoring waits for that: with two workspaces, layer l + 2's scoring would wait
-    # for layer l's gather as well).  The launches of a step are
-    # captured into a CUDA graph (per-kernel launch cost ~1 us instead of ~3 us on a stream)
-    # and the graph is replayed; the allocation still runs on the host every step and must
-    # reproduce the budgets the graph was captured with.
-    ws_score = [sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev) for _ in range(N_SCORE_WS)]
-    ws_sel = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
-    stream = torch.cuda.current_stream(dev)
-    lo_prio, hi_prio = torch.cuda.Stream.priority_range()
-    sel_stream = torch.cuda.Stream(dev, priority=hi_prio)
-    fork = torch.cuda.Event()
-    scored = [torch.cuda.Event() for _ in range(Ls)]
-    pooled = [torch.cuda.Event() for _ in range(Ls)]     # workspace l % N_SCORE_WS read
-    done = torch.cuda.Event()
-
-    def launches(ball, s, kinds=(), every=1, first=0):
-        fork.record(s)
-        sel_stream.wait_event(fork)
-        for l in range(Ls):
-            inp, o = layers[l], outs[l]
-            b = ball[l * wl.Hkv:(l + 1) * wl.Hkv]
-            sg.sgdkv_debug_enable_kernel_timing(kinds if l % every == first % every else ())
-            wsl = ws_score[l % N_SCORE_WS]
-            if l >= N_SCORE_WS:
-                s.wait_event(pooled[l - N_SCORE_WS])   # its workspace read by that compaction
-            sg.sgdkv_score_raw(inp["q"], inp["K"], wl.W, wsl, s)
-            scored[l].record(s)
-            sel_stream.wait_event(scored[l])
-            sg.sgdkv_pool_compact(wsl, wl.pool, inp["K"], inp["V"], b, n_sink, n_recent,
-                                  o["scores"], o["idx"], o["cu"], o["ko"], o["vo"], ws_sel,
-                                  sel_stream)
-            pooled[l].record(sel_stream)
-        done.record(sel_stream)
-        s.wait_event(done)
-
-    def allocate():
-        ball = sg.sgdkv_allocate_budgets(hs, wl.L, T, wl.floor)      # a1 (host)
-        if not np.array_equal(ball, b_all):
-            raise RuntimeError("budget allocation changed between steps")
-        return ball
-
-    def capture(kinds, every=1, first=0):
-        """One step's launches as a CUDA graph; the kernels of `kinds` in every `every`-th
-        layer from layer `first` on are bracketed by timing events."""
-        g = torch.cuda.CUDAGraph()
-        n0 = sg.sgdkv_launch_count()
-        with torch.cuda.graph(g):
-            launches(b_all, torch.cuda.current_stream(dev), kinds, every, first)
-        sg.sgdkv_debug_enable_kernel_timing(())
-        return g, sg.sgdkv_launch_count() - n0
-
-    def drain_timers():
-        return [sg.sgdkv_debug_kernel_timing(kind) for kind in range(len(KERNEL_NAMES))]
-
-    def check(where):
-        st = max(max(sg.sgdkv_last_error(w, stream) for w in ws_score),
-                 sg.sgdkv_last_error(ws_sel, sel_stream))
-        if st != sg.OK:
-            raise RuntimeError(f"device-side error {where}: {sg.status_string(st)}")
-
-    launches(allocate(), stream)                 # one eager step (first-use setup), then graphs
-    torch.cuda.synchronize(dev)
-    check("in the first step")
-    g_warm, _ = capture(())
-    for _ in range(max(args.warmup, 0)):
-        allocate()
-        g_warm.replay()
-    torch.cuda.synchronize(dev)
-    check("during warm-up")
-
-    # Diagnostic window (untimed for the headline): every kernel bracketed by CUDA events,
-    # giving each kernel's share of the step and picking the dominant kernel.
-    drain_timers()
-    diag = [capture(range(len(KERNEL_NAMES)))[0] for _ in range(DIAG_STEPS)]
-    for g in diag:
-        allocate()
-        g.replay()
-    torch.cuda.synchronize(dev)
-    kern = {}
-    for name, (tot_ms, n) in zip(KERNEL_NAMES, drain_timers()):
-        kern[name] = {"launches": n, "us_per_launch": 1e3 * tot_ms / max(n, 1), "ms_total": tot_ms,
-                      "dram_bytes_ncu": measured_traffic(name, wl.name)}
-    del diag
-    kern = {k: v for k, v in kern.items() if v["launches"] > 0}   # no pool kernel at this size
-    all_ms = sum(v["ms_total"] for v in kern.values())
-    for v in kern.values():
-        v["share"] = v["ms_total"] / all_ms if all_ms > 0 else None
-    top_kind = max(range(2), key=lambda k: kern[KERNEL_NAMES[k]]["ms_total"])
-    top = KERNEL_NAMES[top_kind]
-
-    # Timed region: K graphs of one step each.  The dominant kernel is bracketed by two event
-    # nodes in every TIMED_EVERY-th layer (each pair costs about 1 us of step time), starting
-    # one layer later in each successive step so that every layer position is sampled alike;
-    # the events are distinct per graph, so every bracketed launch of the timed region is read.
-    K = args.steps
-    timed = [capture([top_kind], TIMED_EVERY, k) for k in range(K)]
-    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    clocks = ClockSampler(nvsmi_id(local))
-    barrier(world)
-    torch.cuda.synchronize(dev)
-    clocks.start()
-    time.sleep(0.3)                      # let the sampler attach before the timed region
-    start.record(stream)
-    for g, _ in timed:
-        allocate()
-        g.replay()
-    end.record(stream)
-    torch.cuda.synchronize(dev)
-    launches_timed = sum(n for _, n in timed)
-    top_ms, top_n = sg.sgdkv_debug_kernel_timing(top_kind)
-    clk = clocks.stop()
-    barrier(world)
-    check("in the timed region")
-    del timed, g_warm
-    ms = start.elapsed_time(end) / K
-    ms_max = max_over_ranks(ms, world)
+    r = StepRunner(wl, args.frac, Ls, dev)
+    m = r.measure(args.steps, args.warmup, DIAG_STEPS, world, local)
+    ms_max = m["ms_max"]
+    kern = m["kern"]
 
     peaks = measured_peaks()
-    top_us = 1e3 * top_ms / max(top_n, 1)
-    achieved_tf = pass_flops(wl) / (top_us * 1e-6) / 1e12
+    # The timed region lasts well under a second at full clocks, so the dominant pass is
+    # set against the burst bf16 peak (the sustained figure is for seconds-long loops).
+    achieved_tf = pass_flops(wl) / (m["top_us"] * 1e-6) / 1e12
     stage_us = sum(kern[n]["us_per_launch"] for n in KERNEL_NAMES[:3] if n in kern)
     stage_tf = score_flops(wl) / (stage_us * 1e-6) / 1e12
-    bytes_step = sum(path_bytes(wl, o["b"]) for o in outs)
+    bytes_step, rf = roofs(wl, r.outs, ms_max, Ls, peaks)
     value = world * wl.L * Ls / (ms_max * 1e-3)
 
-    dec = None if args.no_decode else run_decode(args, wl, outs, dev, stream, peaks)
+    dec = None if args.no_decode else run_decode(args, wl, r.outs, dev, r.stream, peaks)
 
     e2e = None
     if not args.no_e2e and args.e2e_steps > 0:
-        e2e = run_e2e(args, wl, layers, outs, n_sink, n_recent, dev, world)
+        e2e = run_e2e(args, wl, r.layers, r.outs, r.n_sink, r.n_recent, dev, world)
+    r.free()
+    del r
+    torch.cuda.synchronize(dev)
+    torch.cuda.empty_cache()
+
+    sweep = None
+    if not args.no_sweep and world == 1:      # replicas (N > 1) time the headline only
+        sweep = run_sweep(args, world, local, dev, peaks, skip=(wl.name, args.frac)
+                          if Ls == wl.n_layers else None)
 
     rec = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded N(0,1) K/V/Q with planted sink and salient keys)",
         "config": workload_config(wl, args, world, Ls),
-        "roofline": {"kernel": top, "bound": "tensor", "achieved": achieved_tf,
-                     "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
-                     "frac": achieved_tf / peaks["bf16_sus"],
-                     "traffic": measured_traffic(top, wl.name),
-                     "peak_source": peaks["source"] + " bf16 sustained",
-                     "us_per_launch": top_us, "launches_timed": top_n,
+        "roofline": {"kernel": m["top"], "bound": "tensor", "achieved": achieved_tf,
+                     "peak": peaks["bf16"], "unit": "TFLOP/s",
+                     "frac": achieved_tf / peaks["bf16"],
+                     "traffic": measured_traffic(m["top"], wl.name),
+                     "peak_source": peaks["source"] + " bf16 burst (timed region < 1 s)",
+                     "frac_of_sustained": achieved_tf / peaks["bf16_sus"],
+                     "us_per_launch": m["top_us"], "launches_timed": m["top_n"],
                      "timed_launches": f"every {TIMED_EVERY}th layer of every timed step, "
                                        "rotating by one layer per step",
                      "flops_per_launch": pass_flops(wl)},
         "score_stage": {"us_per_layer": stage_us, "tflops": stage_tf,
-                        "frac": stage_tf / peaks["bf16_sus"]},
+                        "frac": stage_tf / peaks["bf16"]},
         "kernels": {"window": f"{DIAG_STEPS} steps after warm-up, every launch bracketed",
                     **kern},
-        "hbm_path": {"achieved_gbs": bytes_step / (ms_max * 1e-3) / 1e9,
-                     "peak_gbs": peaks["hbm"], "frac": bytes_step / (ms_max * 1e-3) / 1e9 / peaks["hbm"],
-                     "bytes_per_step": bytes_step},
+        **rf,
         "decode_attention": dec,
-        "gpu_launches": int(launches_timed),
+        "gpu_launches": m["launches"],
         "schedule": "each step: budget allocation on the host, then one CUDA-graph launch of "
                     "the step's kernels (the scoring passes on one stream, max-pool + "
                     "selection in one kernel and the gather on a second inside the graph); "
                     "one graph per timed step",
-        "clocks": clk,
+        "clocks": m["clocks"],
         "e2e": e2e,
+        "workloads": sweep,
     }
     return rec
 

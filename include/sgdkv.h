@@ -255,7 +255,9 @@ SGDKV_API sgdkv_status sgdkv_score_static(const void* q_win, const void* K, int3
  *                 addresses directly (cudaHostAlloc, cudaHostRegister).  Only the kept rows
  *                 are read (by the gather), so a cache held in host memory crosses the host
  *                 link for the kept rows alone.
- * scores          device fp32 [Hkv][L], finite and >= 0 (as produced by sgdkv_score)
+ * scores          device fp32 [Hkv][L], finite and >= 0 (as produced by sgdkv_score); -0.0
+ *                 counts as +0.0.  NaN or negative scores are outside the contract: the
+ *                 selection is then unspecified, though every write stays in bounds
  * budgets         HOST int64 [Hkv], n_sink + n_recent <= b_h <= L
  * indices_out     device int32 [sum b_h]: kept positions, head by head
  * cu_seqlens_out  device int32 [Hkv + 1]: cu[0] = 0, cu[h+1] = cu[h] + b_h

@@ -2,8 +2,8 @@
 // tokens, then each head's top (b_h - n_sink - n_recent) middle tokens by score; equal
 // scores are broken by the lower position).
 //
-// Scores are finite and non-negative, so their fp32 bit patterns sort like their values
-// and the threshold search is an exact most-significant-digit radix select on uint32 keys:
+// Scores are finite and non-negative (-0.0 is read as +0.0), so their fp32 bit patterns
+// sort like their values and the threshold search is an exact most-significant-digit radix select on uint32 keys:
 // four passes of 8-bit digits, each a histogram over the middle keys that match the digits
 // fixed so far.  One thread-block cluster works on one KV head: every CTA owns a
 // contiguous slice of the row, builds its histogram in shared memory, and after a cluster
@@ -16,6 +16,8 @@
 // (the four raw planes summed, then the window maximum, Section 3.3), so the max-pool needs
 // no launch of its own.
 #include <cooperative_groups.h>
+
+#include <mutex>
 
 #include "sgdkv_internal.cuh"
 
@@ -78,6 +80,13 @@ struct KeepRule {
   __device__ __forceinline__ bool above(uint32_t u) const { return !none && u > tau; }
   __device__ __forceinline__ bool tie(uint32_t u) const { return !none && u == tau; }
 };
+
+// Radix key of a score: its fp32 bit pattern, with -0.0 read as +0.0 (the two compare
+// equal, and the sign bit would otherwise rank -0.0 above every positive score).
+__device__ __forceinline__ uint32_t score_key(float s) {
+  const uint32_t u = __float_as_uint(s);
+  return u == 0x80000000u ? 0u : u;
+}
 
 // Shared-memory index of the pool buffer: one word of skew per 32, so that the 16 or so
 // consecutive words each thread reads fall into different banks across a warp.
@@ -178,7 +187,7 @@ __device__ __forceinline__ void pool_slice(const PoolSrc& ps, int h, int64_t L, 
     }
   }
 #pragma unroll
-  for (int i = 0; i < PER; ++i) u[i] = i < nv ? __float_as_uint(m[i]) : 0u;
+  for (int i = 0; i < PER; ++i) u[i] = i < nv ? score_key(m[i]) : 0u;
   float* o = ps.out + int64_t(h) * L + p0;
   if (nv == PER && PER % 4 == 0 && (reinterpret_cast<uintptr_t>(o) & 15) == 0) {
 #pragma unroll
@@ -227,7 +236,7 @@ sel_cluster_kernel(const float* __restrict__ scores, HeadTable ht, int csize,
     pool_slice<PER>(ps, h, L, beg, end, p0, u);
   } else if constexpr (PER > 0) {
 #pragma unroll
-    for (int i = 0; i < PER; ++i) u[i] = p0 + i < end ? __float_as_uint(__ldg(row + p0 + i)) : 0u;
+    for (int i = 0; i < PER; ++i) u[i] = p0 + i < end ? score_key(__ldg(row + p0 + i)) : 0u;
   }
 
   uint32_t cand = 0u;                       // PER > 0: bit i = position p0+i is middle
@@ -271,7 +280,7 @@ sel_cluster_kernel(const float* __restrict__ scores, HeadTable ht, int csize,
       } else {
 #pragma unroll 4
         for (int64_t j = mb + tid; j < me; j += kCThreads) {
-          const uint32_t x = __float_as_uint(__ldg(row + j));
+          const uint32_t x = score_key(__ldg(row + j));
           if ((x & hi_mask) == prefix) atomicAdd(&sm.wh[wid][(x >> shift) & 255u], 1u);
         }
       }
@@ -324,7 +333,7 @@ sel_cluster_kernel(const float* __restrict__ scores, HeadTable ht, int csize,
         ++nk;
         continue;
       }
-      const uint32_t x = __float_as_uint(__ldg(row + j));
+      const uint32_t x = score_key(__ldg(row + j));
       nk += kr.above(x);
       nt += kr.tie(x);
     }
@@ -395,7 +404,7 @@ sel_cluster_kernel(const float* __restrict__ scores, HeadTable ht, int csize,
       for (int i = 0; i < kPer; ++i) {
         const int64_t j = q0 + i;
         const bool mid = j < end && !kr.protected_pos(j);
-        x[i] = mid ? __float_as_uint(__ldg(row + j)) : 0u;
+        x[i] = mid ? score_key(__ldg(row + j)) : 0u;
         my_ties += (mid && kr.tie(x[i])) ? 1u : 0u;
       }
       uint32_t round_ties;
@@ -478,36 +487,52 @@ constexpr size_t sel_smem_bytes() {
 }
 
 // Largest cluster size (16 if the device runs it, else the portable 8) for the selection.
+// The kernel's shared-memory and cluster-size attributes belong to the device that is
+// current when they are set, so they are set, and the size found, once per device, under a
+// lock (host threads may launch on several devices at once).
+constexpr int kMaxSelDevices = 64;
+
+template <int PER, bool POOL>
+int probe_cluster_size() {
+  int size = 8;
+  constexpr size_t smem = sel_smem_bytes<PER, POOL>();
+  cudaFuncSetAttribute(sel_cluster_kernel<PER, POOL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       int(smem));
+  if (cudaFuncSetAttribute(sel_cluster_kernel<PER, POOL>,
+                           cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(16, 1, 1);
+    cfg.blockDim = dim3(kCThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = 16;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxPotentialClusterSize(&n, sel_cluster_kernel<PER, POOL>, &cfg) ==
+            cudaSuccess &&
+        n >= 16)
+      size = 16;
+  }
+  cudaGetLastError();   // a refused query leaves the portable size
+  return size;
+}
+
 template <int PER, bool POOL>
 int cluster_size() {
-  static int cached = 0;
-  if (cached == 0) {
-    cached = 8;
-    constexpr size_t smem = sel_smem_bytes<PER, POOL>();
-    cudaFuncSetAttribute(sel_cluster_kernel<PER, POOL>,
-                         cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-    if (cudaFuncSetAttribute(sel_cluster_kernel<PER, POOL>,
-                             cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
-      cudaLaunchConfig_t cfg = {};
-      cfg.gridDim = dim3(16, 1, 1);
-      cfg.blockDim = dim3(kCThreads, 1, 1);
-      cfg.dynamicSmemBytes = smem;
-      cudaLaunchAttribute attr;
-      attr.id = cudaLaunchAttributeClusterDimension;
-      attr.val.clusterDim.x = 16;
-      attr.val.clusterDim.y = 1;
-      attr.val.clusterDim.z = 1;
-      cfg.attrs = &attr;
-      cfg.numAttrs = 1;
-      int n = 0;
-      if (cudaOccupancyMaxPotentialClusterSize(&n, sel_cluster_kernel<PER, POOL>, &cfg) ==
-              cudaSuccess &&
-          n >= 16)
-        cached = 16;
-    }
-    cudaGetLastError();   // a refused query leaves the portable size
+  static std::mutex mu;
+  static int cached[kMaxSelDevices] = {};
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxSelDevices) {
+    cudaGetLastError();
+    return probe_cluster_size<PER, POOL>();      // no slot to cache in: set up every call
   }
-  return cached;
+  std::lock_guard<std::mutex> lock(mu);
+  if (cached[dev] == 0) cached[dev] = probe_cluster_size<PER, POOL>();
+  return cached[dev];
 }
 
 template <int PER, bool POOL>

@@ -15,6 +15,8 @@ from oracle import sgdkv_oracle as O
 from paper_2609_03235_gb300 import configs, synth
 from paper_2609_03235_gb300 import sgdkv as sg
 
+from _guard import guarded
+
 pytestmark = pytest.mark.gpu
 
 
@@ -40,11 +42,12 @@ def _run(dev, q, K, V, budgets):
     qt = synth.to_torch_bf16(q, dev)
     Kt = synth.to_torch_bf16(K, dev) if R else None
     Vt = synth.to_torch_bf16(V, dev) if R else None
-    out = torch.full((Hq, n_tok, 128), float("nan"), dtype=torch.float32, device=dev)
+    g_out = guarded((Hq, n_tok, 128), torch.float32, dev, fill=float("nan"))
     ws = sg.make_decode_workspace(Hq, Hkv, n_tok, R, dev)
-    sg.sgdkv_decode_attention(qt, Kt, Vt, budgets, out, ws)
+    sg.sgdkv_decode_attention(qt, Kt, Vt, budgets, g_out.t, ws)
     torch.cuda.synchronize()
-    return out.cpu().numpy()
+    g_out.check("decode output")
+    return g_out.t.cpu().numpy()
 
 
 def _check(got, q, K, V, budgets):

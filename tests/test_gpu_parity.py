@@ -14,6 +14,8 @@ from oracle import sgdkv_oracle as O
 from paper_2609_03235_gb300 import configs, synth
 from paper_2609_03235_gb300 import sgdkv as sg
 
+from _guard import guarded, check_all
+
 pytestmark = pytest.mark.gpu
 RTOL, ATOL = 2e-3, 1e-5
 
@@ -290,24 +292,56 @@ def test_compact_parity_identical_scores(dev, Hkv, L, n_sink, n_recent, rule, ti
     ws = sg.make_workspace(Hkv, Hkv, L, 32, dev) if L >= 32 else sg.make_workspace(1, 1, 32, 32, dev)
     Kt, Vt = synth.to_torch_bf16(K, dev), synth.to_torch_bf16(V, dev)
     st = torch.from_numpy(scores).to(dev)
-    idx = torch.full((max(total, 1),), -1, dtype=torch.int32, device=dev)
-    cu = torch.full((Hkv + 1,), -1, dtype=torch.int32, device=dev)
-    ko = torch.zeros((max(total, 1), 128), dtype=torch.bfloat16, device=dev)
-    vo = torch.zeros((max(total, 1), 128), dtype=torch.bfloat16, device=dev)
+    g_idx = guarded((total,), torch.int32, dev, fill=-1)
+    g_cu = guarded((Hkv + 1,), torch.int32, dev, fill=-1)
+    g_ko = guarded((total, 128), torch.bfloat16, dev, fill=0)
+    g_vo = guarded((total, 128), torch.bfloat16, dev, fill=0)
+    idx, cu, ko, vo = g_idx.t, g_cu.t, g_ko.t, g_vo.t
     for _ in range(2):       # the same workspace twice in a row
         sg.sgdkv_compact(Kt, Vt, st, b, n_sink, n_recent, idx, cu, ko, vo, ws)
         torch.cuda.synchronize()
         assert sg.sgdkv_last_error(ws) == sg.OK
+        check_all(g_idx, g_cu, g_ko, g_vo)
         e_idx, e_cu = O.select_indices(scores, b, n_sink, n_recent)
         assert np.array_equal(cu.cpu().numpy(), e_cu)
-        assert np.array_equal(idx[:total].cpu().numpy(), e_idx)
+        assert np.array_equal(idx.cpu().numpy(), e_idx)
         e_ko, e_vo = O.gather(K, V, e_idx, e_cu)
-        assert np.array_equal(synth.from_torch_bf16(ko[:total]), e_ko)
-        assert np.array_equal(synth.from_torch_bf16(vo[:total]), e_vo)
+        assert np.array_equal(synth.from_torch_bf16(ko), e_ko)
+        assert np.array_equal(synth.from_torch_bf16(vo), e_vo)
 
 
-def _check_end_to_end(inp, out, budgets, n_sink, n_recent, pool):
-    raw = O.window_scores(inp["q"], inp["K"])
+def test_compact_negative_zero_scores_count_as_zero(dev):
+    """-0.0 compares equal to +0.0: a row of zeros with some -0.0 keeps the lowest middle
+    positions, as the oracle's (score desc, position asc) order does."""
+    Hkv, L = 2, 5000
+    rng = np.random.default_rng(3)
+    scores = np.zeros((Hkv, L), np.float32)
+    scores[:, rng.choice(L, 400, replace=False)] = np.float32(-0.0)
+    scores[1, rng.choice(L, 50, replace=False)] = 0.5
+    K = synth.bf16_round(rng.standard_normal((Hkv, L, 128), dtype=np.float32))
+    V = synth.bf16_round(rng.standard_normal((Hkv, L, 128), dtype=np.float32))
+    b = np.array([300, 200], np.int64)
+    total = int(b.sum())
+    ws = sg.make_workspace(Hkv, Hkv, L, 32, dev)
+    g_idx = guarded((total,), torch.int32, dev, fill=-1)
+    g_cu = guarded((Hkv + 1,), torch.int32, dev, fill=-1)
+    g_ko = guarded((total, 128), torch.bfloat16, dev, fill=0)
+    g_vo = guarded((total, 128), torch.bfloat16, dev, fill=0)
+    sg.sgdkv_compact(synth.to_torch_bf16(K, dev), synth.to_torch_bf16(V, dev),
+                     torch.from_numpy(scores).to(dev), b, 16, 16, g_idx.t, g_cu.t, g_ko.t,
+                     g_vo.t, ws)
+    torch.cuda.synchronize()
+    assert sg.sgdkv_last_error(ws) == sg.OK
+    check_all(g_idx, g_cu, g_ko, g_vo)
+    e_idx, e_cu = O.select_indices(scores, b, 16, 16)
+    assert np.array_equal(g_cu.t.cpu().numpy(), e_cu)
+    assert np.array_equal(g_idx.t.cpu().numpy(), e_idx)
+    assert np.array_equal(e_idx[:b[0]], np.concatenate([np.arange(300 - 16), np.arange(L - 16, L)]))
+
+
+def _check_end_to_end(inp, out, budgets, n_sink, n_recent, pool, raw=None):
+    if raw is None:
+        raw = O.window_scores(inp["q"], inp["K"])
     exp = O.max_pool(raw, pool) if pool > 1 else raw
     got = out["scores"].cpu().numpy()
     ok = _within(got, exp)
@@ -365,12 +399,16 @@ def test_pool_compact_equals_pool_then_compact(dev, Hq, Hkv, L, W, pool, flags_n
     ws_sel = sg.make_workspace(Hq, Hkv, L, W, dev)
     sg.sgdkv_score_raw(q, K, W, ws, flags=flags, head_weights=hw)
 
+    guards = []
+
     def outs():
-        return dict(scores=torch.full((Hkv, L), float("nan"), dtype=torch.float32, device=dev),
-                    idx=torch.full((total,), -1, dtype=torch.int32, device=dev),
-                    cu=torch.full((Hkv + 1,), -1, dtype=torch.int32, device=dev),
-                    ko=torch.zeros((total, 128), dtype=torch.bfloat16, device=dev),
-                    vo=torch.zeros((total, 128), dtype=torch.bfloat16, device=dev))
+        gs = dict(scores=guarded((Hkv, L), torch.float32, dev, fill=float("nan")),
+                  idx=guarded((total,), torch.int32, dev, fill=-1),
+                  cu=guarded((Hkv + 1,), torch.int32, dev, fill=-1),
+                  ko=guarded((total, 128), torch.bfloat16, dev, fill=0),
+                  vo=guarded((total, 128), torch.bfloat16, dev, fill=0))
+        guards.extend(gs.values())
+        return {k: g.t for k, g in gs.items()}
     a, f = outs(), outs()
     sg.sgdkv_pool_raw(ws, Hkv, L, pool, a["scores"], flags=flags)
     sg.sgdkv_compact(K, V, a["scores"], b, n_sink, n_recent, a["idx"], a["cu"], a["ko"],
@@ -379,6 +417,7 @@ def test_pool_compact_equals_pool_then_compact(dev, Hq, Hkv, L, W, pool, flags_n
                           f["ko"], f["vo"], ws_sel, flags=flags)
     torch.cuda.synchronize()
     assert sg.sgdkv_last_error(ws) == sg.OK and sg.sgdkv_last_error(ws_sel) == sg.OK
+    check_all(*guards)
     for k in a:
         if a[k].dtype == torch.bfloat16:
             assert torch.equal(a[k].view(torch.int16), f[k].view(torch.int16)), k
@@ -412,23 +451,51 @@ def test_compress_layer_small(dev):
     _check_end_to_end(inp, out, b, 128, 128, 7)
 
 
-@pytest.mark.parametrize("name", [w.name for w in configs.WORKLOADS])
-def test_full_size_layer(dev, name):
-    """One layer of each workload at full size, in the launch configuration the benchmark
-    times (sgdkv_compress_layer with the model-wide greedy allocation)."""
+def _compress_guarded(q, K, V, b, W, pool, n_sink, n_recent, ws, stream=None):
+    """sgdkv_compress_layer into outputs with guard bands; returns (outputs, guards)."""
+    Hkv, L, d = K.shape
+    total = int(np.sum(b))
+    dev = K.device
+    gs = dict(scores=guarded((Hkv, L), torch.float32, dev, fill=float("nan")),
+              indices=guarded((total,), torch.int32, dev, fill=-1),
+              cu_seqlens=guarded((Hkv + 1,), torch.int32, dev, fill=-1),
+              K_out=guarded((total, d), torch.bfloat16, dev, fill=0),
+              V_out=guarded((total, d), torch.bfloat16, dev, fill=0))
+    out = {k: g.t for k, g in gs.items()}
+    sg.sgdkv_compress_layer(q, K, V, b, W, pool, n_sink, n_recent, out["scores"],
+                            out["indices"], out["cu_seqlens"], out["K_out"], out["V_out"], ws,
+                            stream)
+    return out, list(gs.values())
+
+
+FULL_SIZE_CASES = [(w.name, f) for w in configs.WORKLOADS for f in w.budget_fracs]
+_ORACLE_RAW = {}          # the oracle's raw window scores of one full-size layer, by workload
+
+
+@pytest.mark.parametrize("name,frac", FULL_SIZE_CASES,
+                         ids=[f"{n}-{f}" for n, f in FULL_SIZE_CASES])
+def test_full_size_layer(dev, name, frac):
+    """One layer of each workload at full size, at every total budget the workload is
+    measured with (the 128K Qwen2.5-7B shape at 12.5, 25 and 50 %), in the launch
+    configuration the benchmark times (sgdkv_compress_layer with the model-wide greedy
+    allocation); every output inside guard bands."""
     wl = configs.BY_NAME[name]
     layer = wl.n_layers - 1
     inp = synth.layer_inputs_host(wl, layer)
-    frac = 0.25 if 0.25 in wl.budget_fracs else wl.budget_fracs[0]
     all_b = sg.sgdkv_allocate_budgets(synth.head_scores(wl), wl.L, wl.total_budget(frac), wl.floor)
+    assert int(all_b.sum()) == wl.total_budget(frac)
     b = all_b[layer * wl.Hkv:(layer + 1) * wl.Hkv]
     n_sink, n_recent = configs.sink_recent_split(wl.floor)
     q, K, V = _upload(inp, dev)
     ws = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
-    out = sg.compress_layer_alloc(q, K, V, b, wl.W, wl.pool, n_sink, n_recent, ws)
+    out, guards = _compress_guarded(q, K, V, b, wl.W, wl.pool, n_sink, n_recent, ws)
     torch.cuda.synchronize()
     assert sg.sgdkv_last_error(ws) == sg.OK
-    _check_end_to_end(inp, out, b, n_sink, n_recent, wl.pool)
+    check_all(*guards)
+    if name not in _ORACLE_RAW:
+        _ORACLE_RAW.clear()
+        _ORACLE_RAW[name] = O.window_scores(inp["q"], inp["K"])
+    _check_end_to_end(inp, out, b, n_sink, n_recent, wl.pool, raw=_ORACLE_RAW[name])
     # planted keys (4 sinks + salient) survive whenever the middle budget has room
     g_idx, g_cu = out["indices"].cpu().numpy(), out["cu_seqlens"].cpu().numpy()
     for h in range(wl.Hkv):
