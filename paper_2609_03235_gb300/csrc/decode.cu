@@ -97,6 +97,8 @@ decode_partial_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* 
                       const __nv_bfloat16* __restrict__ Vc, DecodeParams p,
                       float* __restrict__ part) {
   extern __shared__ __align__(128) uint8_t dsm[];
+  // the merge kernel may be scheduled now: its blocks wait for this grid's results
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, t = lane & 3;
   const int cg = blockIdx.x;                             // CTA chunk (grid = chunks)
@@ -276,12 +278,15 @@ decode_partial_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* 
   }
 }
 
-// out[h * nq + r][d] = sum_w 2^(m_w - M) o_w[d] / sum_w 2^(m_w - M) l_w over the head's warp
-// chunks w (zeros for a head without rows).  One block per (head, query row): the largest
-// partial max and the weights 2^(m_w - M) with their normaliser are formed once in shared
-// memory, then four groups of 128 threads (one per column) sum interleaved partials.
+// out[h * nq + r][d] = sum_w 2^(m_w - M) o_w[d] / sum_w 2^(m_w - M) l_w over the head's CTA
+// chunks w (zeros for a head without rows).  One block per (head, query row), two global
+// round trips: every partial's (max, sum) is loaded once (up to two per thread) and kept in
+// registers for the block's maximum, the weights 2^(m_w - M) (to shared memory) and the
+// normaliser; then eight groups of 64 threads (one column pair each) sum the weighted
+// partials w = g, g + 8, ... with all of a thread's loads in flight together.
 constexpr int kDCombThreads = 512;
 constexpr int kDMaxChunks = 1024;              // >= kDTargetChunks + SGDKV_MAX_KV_HEADS
+constexpr int kDCombGroups = kDCombThreads / 64;
 
 __device__ __forceinline__ float block_reduce(float v, bool is_max, float* red) {
 #pragma unroll
@@ -302,40 +307,64 @@ __global__ void __launch_bounds__(kDCombThreads)
 decode_combine_kernel(const float* __restrict__ part, DecodeParams p, float* __restrict__ out) {
   __shared__ float f[kDMaxChunks];
   __shared__ float red[kDCombThreads / 32];
-  __shared__ float osum[kDCombThreads / kD][kD];
+  __shared__ float2 osum[kDCombGroups][kD / 2];
+  static_assert(kDMaxChunks <= 2 * kDCombThreads, "two partials per thread");
   const int h = blockIdx.x / p.nq, r = blockIdx.x % p.nq, tid = threadIdx.x;
   const int w0 = p.wpfx[h], n = min(p.wpfx[h + 1] - w0, kDMaxChunks);
   auto row = [&](int w) { return part + (size_t(w0 + w) * 16 + r) * kDPartStride; };
-  float mx = -INFINITY;
-  for (int w = tid; w < n; w += kDCombThreads) mx = fmaxf(mx, __ldg(row(w) + kD));
-  const float M = block_reduce(mx, true, red);
+  // launched as a programmatic dependent of the partial kernel: the partials are complete
+  // and visible once this returns (a no-op after an ordinary launch)
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  float2 ml[2];
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const int w = tid + k * kDCombThreads;
+    ml[k] = w < n ? __ldcg(reinterpret_cast<const float2*>(row(w) + kD))
+                  : make_float2(-INFINITY, 0.f);
+  }
+  const float M = block_reduce(fmaxf(ml[0].x, ml[1].x), true, red);
   float sl = 0.f;
-  for (int w = tid; w < n; w += kDCombThreads) {
-    const float m = __ldg(row(w) + kD);
-    const float fw = (m == -INFINITY) ? 0.f : ex2f(m - M);
-    f[w] = fw;
-    sl += fw * __ldg(row(w) + kD + 1);
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const int w = tid + k * kDCombThreads;
+    if (w < n) {
+      const float fw = ml[k].x == -INFINITY ? 0.f : ex2f(ml[k].x - M);
+      f[w] = fw;
+      sl += fw * ml[k].y;
+    }
   }
   const float S = block_reduce(sl, false, red);   // its barriers also publish f
-  // eight partials per round, their loads issued before the first is used
-  constexpr int kG = kDCombThreads / kD, kU = 8;
-  const int grp = tid / kD, d = tid % kD;
-  float o = 0.f;
-  for (int w = grp; w < n; w += kG * kU) {
-    float v[kU];
+  const int grp = tid >> 6, cp = tid & 63;       // column pair 2 cp, 2 cp + 1
+  float2 o = make_float2(0.f, 0.f);
+  constexpr int kU = 16;
+  for (int w = grp; w < n; w += kDCombGroups * kU) {
+    float2 v[kU];
 #pragma unroll
-    for (int k = 0; k < kU; ++k) v[k] = w + kG * k < n ? __ldg(row(w + kG * k) + d) : 0.f;
+    for (int k = 0; k < kU; ++k) {
+      const int wk = w + kDCombGroups * k;
+      v[k] = wk < n ? __ldcg(reinterpret_cast<const float2*>(row(wk)) + cp)
+                    : make_float2(0.f, 0.f);
+    }
 #pragma unroll
-    for (int k = 0; k < kU; ++k)
-      if (w + kG * k < n) o += f[w + kG * k] * v[k];
+    for (int k = 0; k < kU; ++k) {
+      const int wk = w + kDCombGroups * k;
+      const float fw = wk < n ? f[wk] : 0.f;
+      o.x += fw * v[k].x;
+      o.y += fw * v[k].y;
+    }
   }
-  osum[grp][d] = o;
+  osum[grp][cp] = o;
   __syncthreads();
-  if (tid < kD) {
-    float O = 0.f;
+  if (tid < kD / 2) {
+    float2 O = make_float2(0.f, 0.f);
 #pragma unroll
-    for (int g = 0; g < kDCombThreads / kD; ++g) O += osum[g][tid];
-    out[(size_t(h) * p.nq + r) * kD + tid] = S > 0.f ? O / S : 0.f;
+    for (int g = 0; g < kDCombGroups; ++g) {
+      O.x += osum[g][tid].x;
+      O.y += osum[g][tid].y;
+    }
+    const float inv = S > 0.f ? 1.f / S : 0.f;
+    *reinterpret_cast<float2*>(out + (size_t(h) * p.nq + r) * kD + 2 * tid) =
+        make_float2(O.x * inv, O.y * inv);
   }
 }
 
@@ -396,8 +425,21 @@ cudaError_t launch_decode(const __nv_bfloat16* q, const __nv_bfloat16* Kc,
     note_launches(1);
   }
   {
+    // programmatic dependent launch: the merge blocks are scheduled while the partial
+    // kernel runs (they fit beside its CTAs) and start their work as soon as it completes
     KernelTimer tc(SGDKV_KERNEL_DECODE, stream);
-    decode_combine_kernel<<<unsigned(Hkv * p.nq), kDCombThreads, 0, stream>>>(part, p, out);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(Hkv * p.nq), 1, 1);
+    cfg.blockDim = dim3(kDCombThreads, 1, 1);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr.val.programmaticStreamSerializationAllowed = nchunks > 0 ? 1 : 0;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, decode_combine_kernel, static_cast<const float*>(part), p, out);
+    if (e != cudaSuccess) return e;
     note_launches(1);
   }
   return cudaGetLastError();

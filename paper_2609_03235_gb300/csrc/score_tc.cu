@@ -323,6 +323,19 @@ __device__ __forceinline__ float hsum(uint64_t a, uint64_t b) {
   return (a0 + a1) + (b0 + b1);
 }
 
+// Tile ids handed between roles through shared memory: explicit shared-space accesses (a
+// volatile access through a generic pointer compiles to a system-scope load), ordered by
+// the mbarrier arrive (release) and wait (acquire) around them.
+__device__ __forceinline__ int ld_tile(const volatile int* p) {
+  int v;
+  asm volatile("ld.volatile.shared.s32 %0, [%1];" : "=r"(v) : "r"(smem_u32((const void*)p)) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_tile(volatile int* p, int v) {
+  asm volatile("st.volatile.shared.s32 [%0], %1;" ::"r"(smem_u32((const void*)p)), "r"(v) : "memory");
+}
+
+// ---------------------------------------------------------------------------------------
 // ---------------------------------------------------------------------------------------
 // Shared pieces of both passes
 // ---------------------------------------------------------------------------------------
@@ -437,11 +450,11 @@ __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMa
     if (claim < uint32_t(p.T)) next = atomicAdd(counter, 1u);
     if (!bwait(bar_kempty(s, st), (use & 1) ^ 1, ab, p.wait_ns, status)) break;
     if (tile >= uint32_t(p.T)) {
-      s.stile[st] = -1;
+      st_tile(s.stile + st, -1);
       mbar_arrive(bar_kfull(s, st));            // releases the id; no copy in flight
       break;
     }
-    s.stile[st] = int(tile);
+    st_tile(s.stile + st, int(tile));
     mbar_expect_tx(bar_kfull(s, st), kStageBytes);
     const int row = int(int64_t(h) * p.L + int64_t(tile) * kTileKeys);
     for (int c = 0; c < 2; ++c) {
@@ -482,7 +495,7 @@ __device__ bool mma_start(const Smem& s, const TcParams& p, uint32_t* status) {
 // epilogue's loop: both arrivals are made here.
 __device__ __forceinline__ void publish_slot(const Smem& s, int slot, int tile, uint32_t leader) {
   if (!leader) return;
-  s.utile[slot] = tile;
+  st_tile(s.utile + slot, tile);
   if (tile < 0) mbar_arrive2(bar_tfull(s, slot));
   else mbar_arrive(bar_tfull(s, slot));
 }
@@ -587,7 +600,7 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
       const int st = n % p.nstages;
       if (!(ok = wwait(bar_kfull(s, st), (n / p.nstages) & 1, ab, p.wait_ns, ws.status))) break;
       tc_fence_after();
-      const int tile = s.stile[st];
+      const int tile = ld_tile(s.stile + st);
       const uint32_t k_lo = desc_lo(smem_u32(s.k + st * kStageBytes));
       const int ph = n % NB;
 #pragma unroll
@@ -621,7 +634,7 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
       for (int c = 0;; ++c) {
         if (!bwait(tf, c & 1, ab, p.wait_ns, ws.status)) break;
         tc_fence_after();
-        const int tile = s.utile[wi];
+        const int tile = ld_tile(s.utile + wi);
         if (tile < 0) break;                             // no more tiles
         auto release = [&] {
           tc_fence_before();
@@ -744,7 +757,7 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
       const int st = n % p.nstages;
       if (!(ok = wwait(bar_kfull(s, st), (n / p.nstages) & 1, ab, p.wait_ns, ws.status))) break;
       tc_fence_after();
-      const int tile = s.stile[st];
+      const int tile = ld_tile(s.stile + st);
       const uint32_t k_lo = desc_lo(smem_u32(s.k + st * kStageBytes));
       for (int c = 0; c < nch; ++c) {
         const int u = n * nch + c, slot = u & 1;
@@ -828,7 +841,7 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
         const int u = n * nch + c, slot = u & 1;
         if (!(ok = bwait(bar_tfull(s, slot), (u >> 1) & 1, ab, p.wait_ns, ws.status))) break;
         tc_fence_after();
-        const int tile = s.utile[slot];
+        const int tile = ld_tile(s.utile + slot);
         if (tile < 0) {
           ok = false;                              // no more tiles
           break;

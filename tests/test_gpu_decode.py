@@ -114,3 +114,29 @@ def test_decode_full_size_layer(dev):
     b = np.asarray(all_b[(wl.n_layers - 1) * wl.Hkv: wl.n_layers * wl.Hkv], np.int64)
     q, K, V = _case(wl.Hq, wl.Hkv, 1, b, seed=77, q_scale=2.0)
     _check(_run(dev, q, K, V, b), q, K, V, b)
+
+
+def test_decode_reuses_its_workspace(dev):
+    """One workspace through several calls of different budgets, eager and captured into a
+    CUDA graph (replayed twice): every call gives the oracle's output."""
+    ws = sg.make_decode_workspace(28, 4, 1, 20000, dev)
+    cases = [(28, 4, [1250, 700, 2400, 256], 1), (28, 4, [0, 5000, 3, 9000], 2),
+             (28, 4, [20000, 0, 0, 0], 3)]
+    for Hq, Hkv, budgets, seed in cases:
+        b = np.asarray(budgets, np.int64)
+        q, K, V = _case(Hq, Hkv, 1, b, seed=seed)
+        qt = synth.to_torch_bf16(q, dev)
+        Kt, Vt = synth.to_torch_bf16(K, dev), synth.to_torch_bf16(V, dev)
+        for graph in (False, True):
+            g_out = guarded((Hq, 1, 128), torch.float32, dev, fill=float("nan"))
+            if graph:
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g):
+                    sg.sgdkv_decode_attention(qt, Kt, Vt, b, g_out.t, ws)
+                for _ in range(2):
+                    g.replay()
+            else:
+                sg.sgdkv_decode_attention(qt, Kt, Vt, b, g_out.t, ws)
+            torch.cuda.synchronize()
+            g_out.check("decode output")
+            _check(g_out.t.cpu().numpy(), q, K, V, b)
