@@ -197,17 +197,17 @@ KERNEL_NAMES = ("score_pass1_tc", "score_pass2_tc", "maxpool_sum_kernel", "sel_c
 # DRAM traffic per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one ncu capture
 # of the 128K-context Qwen2.5-7B layer (28 query / 4 KV heads, W=64), keyed by the SHA-256 of
 # the kernel source it was taken on; a source that has changed since reads as null.
-_SCORE_SHA = "e7936773fbe7ce70c3b7e0ac5c4f49450047f96a7e980040dce6593adc033e28"
-_SELECT_SHA = "95ec997644c3fdfdf93a0671515bfdb607f37f72d5ada6e648711d459661f0be"
+_SCORE_SHA = "218010898d786a9c51710ce02ceb32f9c950feb48ba308be71347377a828ab0b"
+_SELECT_SHA = "e9c450f92c12a8c8d98c4432080adc8d741f5023d734eb630f5cd4f1e976c906"
 MEASURED_TRAFFIC = {
     ("score_pass1_tc", "c3_qwen25_7b_L128k"):
-        {"bytes": 134755072 + 3629568, "source": "score_tc.cu", "sha256": _SCORE_SHA},
+        {"bytes": 134759168 + 3032832, "source": "score_tc.cu", "sha256": _SCORE_SHA},
     ("score_pass2_tc", "c3_qwen25_7b_L128k"):
-        {"bytes": 135312896 + 4008448, "source": "score_tc.cu", "sha256": _SCORE_SHA},
+        {"bytes": 135322112 + 3761664, "source": "score_tc.cu", "sha256": _SCORE_SHA},
     ("sel_cluster_kernel", "c3_qwen25_7b_L128k"):
-        {"bytes": 8444416 + 0, "source": "select.cu", "sha256": _SELECT_SHA},
+        {"bytes": 8448768 + 0, "source": "select.cu", "sha256": _SELECT_SHA},
     ("gather_kernel", "c3_qwen25_7b_L128k"):
-        {"bytes": 40768768 + 1776896, "source": "select.cu", "sha256": _SELECT_SHA},
+        {"bytes": 40770816 + 400896, "source": "select.cu", "sha256": _SELECT_SHA},
 }
 
 

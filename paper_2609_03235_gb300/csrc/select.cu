@@ -11,7 +11,9 @@
 // peers through distributed shared memory) and picks the same digit.  The threshold tau and the number of keys equal to tau to keep
 // (lowest positions first) follow.  The same kernel then counts kept positions per slice,
 // exchanges the counts through distributed shared memory, and writes every slice's kept
-// positions, ascending, at their final offsets.  A second kernel copies the kept K/V rows.
+// positions, ascending, at their final offsets.  The kept K/V rows are copied by the
+// selection kernel itself when its CTAs span at least kCopyMinCtas SMs (each CTA copies its
+// slice's rows), else by a second kernel.
 // With a pool source the selection kernel first forms its slice's pooled scores itself
 // (the four raw planes summed, then the window maximum, Section 3.3), so the max-pool needs
 // no launch of its own.
@@ -200,6 +202,15 @@ __device__ __forceinline__ void pool_slice(const PoolSrc& ps, int h, int64_t L, 
   }
 }
 
+// K/V rows to copy from inside the selection kernel (K == nullptr: none; the gather kernel
+// copies them instead).
+struct RowCopy {
+  const uint4* K;
+  const uint4* V;
+  uint4* Ko;
+  uint4* Vo;
+};
+
 // One cluster per KV head (grid = Hkv * csize, cluster = csize CTAs).  Control flow is
 // uniform across a cluster, so every CTA reaches every cluster barrier.
 // PER > 0: each thread holds PER consecutive positions of its CTA's slice in registers for
@@ -210,7 +221,7 @@ template <int PER, bool POOL>
 __global__ void __launch_bounds__(kCThreads)
 sel_cluster_kernel(const float* __restrict__ scores, HeadTable ht, int csize,
                    int32_t* __restrict__ indices_out, int32_t* __restrict__ cu_out,
-                   uint32_t* __restrict__ status, PoolSrc ps) {
+                   uint32_t* __restrict__ status, PoolSrc ps, RowCopy rc) {
   static_assert(!POOL || PER > 0, "inline pooling needs register-resident slices");
   cg::cluster_group cluster = cg::this_cluster();
   __shared__ SelShared sm;
@@ -394,6 +405,37 @@ sel_cluster_kernel(const float* __restrict__ scores, HeadTable ht, int csize,
       if (out + i < out_end) indices_out[out + i] = stage[i];
       else record_error(status, SGDKV_ERR_INTERNAL);
     }
+    if (rc.K) {
+      // ---- the slice's kept K and V rows, copied here (16 threads per 256-byte row, two
+      // rows per thread in flight; read and written once: streaming loads and stores)
+      constexpr uint32_t kRowsPerPass = kCThreads / 16;
+      const int part = tid & 15;
+      const int64_t hrow = int64_t(h) * L;
+      const uint32_t nk = kept < uint32_t(kCThreads * PER) ? kept : uint32_t(kCThreads * PER);
+      for (uint32_t i0 = uint32_t(tid >> 4); i0 < nk; i0 += 2 * kRowsPerPass) {
+        const uint32_t i1 = i0 + kRowsPerPass;
+        const bool ok0 = out + i0 < out_end, ok1 = i1 < nk && out + i1 < out_end;
+        uint4 k0, v0, k1, v1;
+        if (ok0) {
+          const int64_t src = (hrow + stage[i0]) * 16 + part;
+          k0 = __ldcs(rc.K + src);
+          v0 = __ldcs(rc.V + src);
+        }
+        if (ok1) {
+          const int64_t src = (hrow + stage[i1]) * 16 + part;
+          k1 = __ldcs(rc.K + src);
+          v1 = __ldcs(rc.V + src);
+        }
+        if (ok0) {
+          __stcs(rc.Ko + int64_t(out + i0) * 16 + part, k0);
+          __stcs(rc.Vo + int64_t(out + i0) * 16 + part, v0);
+        }
+        if (ok1) {
+          __stcs(rc.Ko + int64_t(out + i1) * 16 + part, k1);
+          __stcs(rc.Vo + int64_t(out + i1) * 16 + part, v1);
+        }
+      }
+    }
   } else {
     // ---- ordered write, rounds of kRound positions -------------------------------------
     for (int64_t r0 = beg; r0 < end; r0 += kRound) {
@@ -538,7 +580,7 @@ int cluster_size() {
 template <int PER, bool POOL>
 cudaError_t launch_select(const float* scores, const HeadTable& ht, int csize,
                           int32_t* indices_out, int32_t* cu_out, uint32_t* status,
-                          const PoolSrc& ps, cudaStream_t stream) {
+                          const PoolSrc& ps, const RowCopy& rc, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(unsigned(ht.Hkv * csize), 1, 1);
   cfg.blockDim = dim3(kCThreads, 1, 1);
@@ -552,7 +594,7 @@ cudaError_t launch_select(const float* scores, const HeadTable& ht, int csize,
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, sel_cluster_kernel<PER, POOL>, scores, ht, csize,
-                            indices_out, cu_out, status, ps);
+                            indices_out, cu_out, status, ps, rc);
 }
 
 // Positions per thread of the selection kernel for rows of length L: slices of up to 32
@@ -568,21 +610,34 @@ int pick_per(int64_t L, int* csize) {
   return 0;
 }
 
+// The selection copies the kept K/V rows itself when its CTAs span at least this many SMs:
+// each CTA moves its slice's rows with ordinary loads and stores, so on fewer SMs the copy
+// is slower than the gather kernel's, which spreads over the whole GPU (measured on the
+// benchmark's two-stream step: 4 KV heads, 64 CTAs, 1.2 % slower; 8 KV heads, 128 CTAs,
+// 4.7 % faster).
+constexpr int kCopyMinCtas = 128;
+
+// rc: the rows to copy when the selection keeps its slices in registers and spans at least
+// kCopyMinCtas CTAs (then *copied is set); otherwise the gather kernel copies them.
 template <bool POOL>
 cudaError_t dispatch_select(const float* scores, const HeadTable& ht, int32_t* indices_out,
                             int32_t* cu_out, uint32_t* status, const PoolSrc& ps,
-                            cudaStream_t stream) {
+                            const RowCopy& rc_in, bool* copied, cudaStream_t stream) {
   int cs = 0;
-  switch (pick_per<POOL>(ht.L, &cs)) {
+  const int per = pick_per<POOL>(ht.L, &cs);
+  *copied = per > 0 && rc_in.K != nullptr && ht.Hkv * cs >= kCopyMinCtas;
+  const RowCopy rc = *copied ? rc_in : RowCopy{nullptr, nullptr, nullptr, nullptr};
+  switch (per) {
     case 8:
-      return launch_select<8, POOL>(scores, ht, cs, indices_out, cu_out, status, ps, stream);
+      return launch_select<8, POOL>(scores, ht, cs, indices_out, cu_out, status, ps, rc, stream);
     case 16:
-      return launch_select<16, POOL>(scores, ht, cs, indices_out, cu_out, status, ps, stream);
+      return launch_select<16, POOL>(scores, ht, cs, indices_out, cu_out, status, ps, rc, stream);
     case 32:
-      return launch_select<32, POOL>(scores, ht, cs, indices_out, cu_out, status, ps, stream);
+      return launch_select<32, POOL>(scores, ht, cs, indices_out, cu_out, status, ps, rc, stream);
     default:
       if (POOL) return cudaErrorInvalidValue;   // callers check compact_pools_inline
-      return launch_select<0, false>(scores, ht, cs, indices_out, cu_out, status, ps, stream);
+      return launch_select<0, false>(scores, ht, cs, indices_out, cu_out, status, ps,
+                                     RowCopy{nullptr, nullptr, nullptr, nullptr}, stream);
   }
 }
 
@@ -594,17 +649,24 @@ cudaError_t launch_compact(const __nv_bfloat16* K, const __nv_bfloat16* V,
                            int64_t total_rows, const Ws& ws, cudaStream_t stream,
                            const PoolSrc* pool_src) {
   cudaError_t e;
+  bool copied = false;
+  const RowCopy rc = total_rows > 0
+                         ? RowCopy{reinterpret_cast<const uint4*>(K),
+                                   reinterpret_cast<const uint4*>(V),
+                                   reinterpret_cast<uint4*>(K_out), reinterpret_cast<uint4*>(V_out)}
+                         : RowCopy{nullptr, nullptr, nullptr, nullptr};
   {
     KernelTimer t(SGDKV_KERNEL_SELECT, stream);
     if (pool_src)
-      e = dispatch_select<true>(pool_src->out, ht, indices_out, cu_out, ws.status, *pool_src,
-                                stream);
+      e = dispatch_select<true>(pool_src->out, ht, indices_out, cu_out, ws.status, *pool_src, rc,
+                                &copied, stream);
     else
-      e = dispatch_select<false>(scores, ht, indices_out, cu_out, ws.status, PoolSrc{}, stream);
+      e = dispatch_select<false>(scores, ht, indices_out, cu_out, ws.status, PoolSrc{}, rc,
+                                 &copied, stream);
   }
   if (e != cudaSuccess) return e;
   note_launches(1);
-  if (total_rows > 0) {
+  if (total_rows > 0 && !copied) {
     KernelTimer tg(SGDKV_KERNEL_GATHER, stream);
     note_launches(1);
     int64_t blocks = ceil_div(total_rows * 16, 256);

@@ -266,6 +266,8 @@ COMPACT_CASES = [
     (1, 1, 0, 0, "full"),
     (2, 200000, 64, 64, "random"),    # 16 positions per thread
     (1, 600000, 64, 64, "random"),    # streaming selection: several ordered-write rounds
+    (8, 5000, 16, 16, "random"),      # 8 x 16 CTAs: the selection copies the rows itself
+    (12, 3001, 0, 32, "quarter"),     # the same, ragged slices
 ]
 
 
@@ -377,6 +379,7 @@ POOL_COMPACT_CASES = [
     (28, 4, 20000, 64, 1, "sum"),     # no pooling (radius 0)
     (2, 1, 300000, 16, 7, "sum"),     # 32 positions per thread
     (2, 1, 600000, 16, 7, "sum"),     # rows too long for register slices: two kernels
+    (64, 8, 3000, 32, 7, "sum"),      # 8 KV heads: rows copied inside the selection kernel
 ]
 
 
@@ -559,15 +562,17 @@ def test_layers_on_two_streams(dev):
         _check_end_to_end(inp, out, b, 128, 128, 7)
 
 
-def test_compact_reads_kv_from_pinned_host_memory(dev):
+@pytest.mark.parametrize("Hkv", [3, 8])
+def test_compact_reads_kv_from_pinned_host_memory(dev, Hkv):
     """K and V of sgdkv_compact (and V of sgdkv_compress_layer) may be pinned host memory:
-    the gather reads the kept rows across the host link; outputs bit-exact."""
-    rng = np.random.default_rng(11)
-    Hkv, L = 3, 3000
+    the kept rows are read across the host link (by the gather kernel with 3 KV heads, by
+    the selection kernel itself with 8); outputs bit-exact."""
+    rng = np.random.default_rng(11 + Hkv)
+    L = 3000
     scores = rng.random((Hkv, L)).astype(np.float32)
     K = synth.bf16_round(rng.standard_normal((Hkv, L, 128), dtype=np.float32))
     V = synth.bf16_round(rng.standard_normal((Hkv, L, 128), dtype=np.float32))
-    b = np.array([700, 64, 3000], np.int64)
+    b = np.array(([700, 64, 3000] * 3)[:Hkv], np.int64)
     total = int(b.sum())
     Kh = synth.to_torch_bf16(K, "cpu").pin_memory()
     Vh = synth.to_torch_bf16(V, "cpu").pin_memory()
