@@ -383,6 +383,27 @@ class StepRunner:
         all_ms = sum(v["ms_total"] for v in kern.values())
         for v in kern.values():
             v["share"] = v["ms_total"] / all_ms if all_ms > 0 else None
+        # the compaction kernels against their roofs: the selection's algorithmic bytes are
+        # the raw planes it pools (16 B per key) and the pooled scores and indices it writes;
+        # the gather's, the kept rows read and written plus their indices
+        wl, hbm = self.wl, measured_peaks()["hbm"]
+        kept = sum(int(o["b"].sum()) for o in self.outs) / max(self.Ls, 1)
+        copied = "gather_kernel" not in kern     # the selection copied the rows itself
+        roof_bytes = {"sel_cluster_kernel": wl.Hkv * wl.L * (16 + 4) + kept * 4 +
+                      (kept * 4 * wl.d * 2 if copied else 0),
+                      "gather_kernel": kept * (4 * wl.d * 2 + 4)}
+        bound = {"sel_cluster_kernel": "latency (cluster barriers and histogram exchange; "
+                                       "inputs L2-resident)" +
+                                       ("; plus the HBM copy of the kept rows" if copied else ""),
+                 "gather_kernel": "hbm"}
+        for name, byts in roof_bytes.items():
+            if name in kern:
+                gbs = byts / (kern[name]["us_per_launch"] * 1e-6) / 1e9
+                kern[name]["roofline"] = {"bound": bound[name], "bytes_per_launch": byts,
+                                          "achieved_gbs": gbs, "peak_gbs": hbm,
+                                          "frac_of_hbm": gbs / hbm,
+                                          "note": "live duration, sharing SMs with the "
+                                                  "scoring stream"}
         top_kind = max(range(2), key=lambda k: kern[KERNEL_NAMES[k]]["ms_total"])
         timed = [self.capture([top_kind], TIMED_EVERY, k) for k in range(steps)]
         start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
