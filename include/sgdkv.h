@@ -319,7 +319,13 @@ SGDKV_API sgdkv_status sgdkv_pool_compact(const void* score_workspace, size_t sc
  * Arithmetic: logits with bf16 products and fp32 sums, softmax in fp32 (log2 units), the
  * weights rounded to bf16 for the value sum, normalised by the sum of the rounded weights;
  * the output is a convex combination of the head's value rows, within 2^-8 max|v| of the
- * exact one.  Asynchronous on stream.  Errors: INVALID_ARG, UNSUPPORTED, WORKSPACE, CUDA.
+ * exact one.  Asynchronous on stream.  Two kernels, both launched as programmatic dependents
+ * of what precedes them on the stream: a call placed right after another decode call (one
+ * per layer, say) starts streaming its cache while the previous call's merge runs, so its
+ * q, K_cache, V_cache and budgets-derived layout must not be outputs of that previous call
+ * (out of one call is never an input of the next in a decode step); it rewrites the shared
+ * workspace only after the previous call has completed.  Errors: INVALID_ARG, UNSUPPORTED,
+ * WORKSPACE, CUDA.
  */
 SGDKV_API size_t sgdkv_decode_workspace_bytes(int32_t Hq, int32_t Hkv, int32_t n_tok, int32_t d,
                                               int64_t total_rows);

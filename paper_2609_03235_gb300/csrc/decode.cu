@@ -17,7 +17,10 @@
 // accumulators.  The row sums are taken over the rounded weights, so every output is a
 // convex combination of the head's value rows.  The four warps of a CTA merge their (max,
 // sum, 128 sums) per query row in shared memory into one partial per CTA chunk; a second
-// kernel merges a head's partials.
+// kernel merges a head's partials.  Both kernels are programmatic dependents of what
+// precedes them: the merge's blocks wait in hardware for the partials, and the partial
+// kernel of a call that follows another decode call streams its cache while the previous
+// merge runs, writing its partials only after that merge has completed.
 #include "sgdkv_internal.cuh"
 
 namespace sgdkv {
@@ -256,6 +259,9 @@ decode_partial_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* 
     r1[kD + 1] = l1;
   }
   __syncthreads();
+  // launched as a programmatic dependent of the previous call's merge: the streaming above
+  // overlapped it, and the partials it reads are rewritten only once it has completed
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int d = threadIdx.x;                             // kDWarps * 32 == kD columns
   for (int r = 0; r < p.nq; ++r) {
     float M = -INFINITY;
@@ -312,6 +318,9 @@ decode_combine_kernel(const float* __restrict__ part, DecodeParams p, float* __r
   const int h = blockIdx.x / p.nq, r = blockIdx.x % p.nq, tid = threadIdx.x;
   const int w0 = p.wpfx[h], n = min(p.wpfx[h + 1] - w0, kDMaxChunks);
   auto row = [&](int w) { return part + (size_t(w0 + w) * 16 + r) * kDPartStride; };
+  // the next call's partial kernel may be scheduled now (it writes the partials only after
+  // this grid has completed)
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   // launched as a programmatic dependent of the partial kernel: the partials are complete
   // and visible once this returns (a no-op after an ordinary launch)
   asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -419,9 +428,21 @@ cudaError_t launch_decode(const __nv_bfloat16* q, const __nv_bfloat16* Kc,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   if (nchunks > 0) {
+    // programmatic dependent launch as well: back-to-back calls (one per layer) overlap,
+    // this call's streaming with the previous call's merge
     KernelTimer tk(SGDKV_KERNEL_DECODE, stream);
-    decode_partial_kernel<<<unsigned(nchunks), kDWarps * 32, smem, stream>>>(
-        q, Kc, Vc, p, part);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(nchunks), 1, 1);
+    cfg.blockDim = dim3(kDWarps * 32, 1, 1);
+    cfg.dynamicSmemBytes = size_t(smem);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr.val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, decode_partial_kernel, q, Kc, Vc, p, part);
+    if (e != cudaSuccess) return e;
     note_launches(1);
   }
   {
