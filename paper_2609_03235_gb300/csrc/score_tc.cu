@@ -54,7 +54,7 @@ constexpr int kMaxStages = 8;
 constexpr int kTmemSlots = 4;                     // TMEM slots (pass 1: 4 x 128 columns, pass 2: 2 x 256)
 constexpr int kNumBars = 2 * kMaxStages + 2 * kTmemSlots + 3;   // kfull kempty tfull tempty qfull drain never
 constexpr int kCtlBytes = 512;                    // barriers, TMEM address, abort flag, tile ids
-static_assert(kNumBars * 8 + 8 + (kMaxStages + kTmemSlots) * 4 <= kCtlBytes, "control block");
+static_assert(kNumBars * 8 + 8 + (kMaxStages + kTmemSlots + 1) * 4 <= kCtlBytes, "control block");
 constexpr int kSmemLimit = 232448;                // opt-in dynamic shared memory per CTA
 constexpr int kQBoxRows = 32;                     // TMA box height for Q rows (pass 2)
 constexpr uint32_t kFlagStallMma = 1u;            // test hook: MMA thread waits on `never`
@@ -347,6 +347,7 @@ struct Smem {
   int* abort_flag;
   volatile int* stile; // [kMaxStages] key tile held by each K stage (-1: no more tiles)
   volatile int* utile; // [kTmemSlots] key tile whose products fill each TMEM slot (-1: done)
+  volatile uint32_t* claims;   // the producer's last claim (see produce)
   float* tail;         // pass 2: -lse2[kMaxRows] (16-byte aligned)
   int qrows;
 };
@@ -362,6 +363,7 @@ __device__ __forceinline__ Smem carve(uint8_t* base, int qrows, int nstages) {
   s.abort_flag = reinterpret_cast<int*>(ctl + kNumBars * 8 + 4);
   s.stile = reinterpret_cast<int*>(ctl + kNumBars * 8 + 8);
   s.utile = s.stile + kMaxStages;
+  s.claims = reinterpret_cast<volatile uint32_t*>(s.utile + kTmemSlots);
   s.tail = reinterpret_cast<float*>(ctl + kCtlBytes);
   return s;
 }
@@ -419,28 +421,43 @@ __device__ __forceinline__ void teardown(uint32_t tmem) {
   }
 }
 
-// TMA producer (one thread): Q rows of head h once, then key tiles of head h claimed one
-// at a time from the head's counter (shared by the head's CTAs; the next claim is made while
-// the current tile's stage is awaited) until none are left; the stage after the last one
-// carries tile id -1 and no data.  second (pass 2): pass 2 reads the keys pass 1 has just
+// Producer thread, once its last claim has returned: the head's last CTA to get here resets
+// the head's tile counter (and the finish count) for the next launch.
+__device__ __forceinline__ void finish_claims(uint32_t* counter, uint32_t* finished, int cph) {
+  __threadfence();
+  if (atomicAdd(finished, 1u) == uint32_t(cph - 1)) {
+    atomicExch(counter, 0u);
+    atomicExch(finished, 0u);
+  }
+}
+
+// TMA producer (one thread): key tiles of head h claimed one at a time from the head's
+// counter (shared by the head's CTAs; `first` is the claim made at kernel entry, the next
+// claim is made while the current tile's stage is awaited) until none are left, and the Q
+// rows of head h once, right after the first key tile (which comes from HBM, the Q rows from
+// L2); the stage after the last tile carries tile id -1 and no data.  Once its last claim
+// has returned the thread counts the CTA's claims finished (finish_claims), while the CTA's
+// last tiles are still being consumed.  second (pass 2): pass 2 reads the keys pass 1 has just
 // read, so it takes a head's tiles from the last one down, starting on the tiles pass 1
 // loaded last, which are still in L2, and loads them evict-first (nothing reads them after
 // pass 2), so that its misses do not push out the tiles it has yet to reach.
 __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMap* tm_k,
-                        const TcParams& p, int h, uint32_t* counter, bool load_q, bool second,
-                        uint32_t* status) {
+                        const TcParams& p, int h, uint32_t* counter, uint32_t* finished,
+                        uint32_t first, bool second, uint32_t* status) {
   volatile int* ab = s.abort_flag;
-  if (load_q) {
+  bool q_issued = false;
+  auto load_q = [&] {
     mbar_expect_tx(bar_qfull(s), uint32_t(2 * s.qrows * 128));
     for (int c = 0; c < 2; ++c)
       for (int b = 0; b < s.qrows / kQBoxRows; ++b)
         tma_load_2d(smem_u32(s.q + (c * s.qrows + b * kQBoxRows) * 128), tm_q, 64 * c,
                     h * p.GW + kQBoxRows * b, bar_qfull(s));
-  }
+    q_issued = true;
+  };
   int issued[kMaxStages];
   for (int i = 0; i < kMaxStages; ++i) issued[i] = 0;
   const uint64_t k_policy = second ? l2_evict_first() : 0;
-  uint32_t next = atomicAdd(counter, 1u);       // the next claim overlaps the stage wait
+  uint32_t next = first;                        // the next claim overlaps the stage wait
   for (int n = 0;; ++n) {
     const int st = n % p.nstages;
     const int use = n / p.nstages;
@@ -452,6 +469,7 @@ __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMa
     if (tile >= uint32_t(p.T)) {
       st_tile(s.stile + st, -1);
       mbar_arrive(bar_kfull(s, st));            // releases the id; no copy in flight
+      if (!q_issued) load_q();
       break;
     }
     st_tile(s.stile + st, int(tile));
@@ -465,11 +483,16 @@ __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMa
         tma_load_2d(dst, tm_k, 64 * c, row, bar_kfull(s, st));
     }
     issued[st] = use + 1;
+    if (!q_issued) load_q();
   }
+  // The claim still in flight after an abort is waited for by this store; then every claim
+  // of the CTA has reached the counter.
+  *s.claims = next;
+  finish_claims(counter, finished, p.cph);
   if (*ab) {
     // Drain: every copy this thread started must have landed before the CTA exits.
     volatile int no_abort = 0;
-    if (load_q) bwait(bar_qfull(s), 0, &no_abort, kDrainNs, status);
+    if (q_issued) bwait(bar_qfull(s), 0, &no_abort, kDrainNs, status);
     for (int st = 0; st < p.nstages; ++st)
       if (issued[st] > 0)
         bwait(bar_kfull(s, st), (issued[st] - 1) & 1, &no_abort, kDrainNs, status);
@@ -500,15 +523,6 @@ __device__ __forceinline__ void publish_slot(const Smem& s, int slot, int tile, 
   else mbar_arrive(bar_tfull(s, slot));
 }
 
-// End of a pass, thread 0 after the CTA's last barrier: the head's last CTA to finish resets
-// the head's tile counter (and the finish count) for the next launch.
-__device__ __forceinline__ void finish_claims(uint32_t* counter, uint32_t* finished, int cph) {
-  __threadfence();
-  if (atomicAdd(finished, 1u) == uint32_t(cph - 1)) {
-    atomicExch(counter, 0u);
-    atomicExch(finished, 0u);
-  }
-}
 
 // MMA warp, after an abort: a commit arrives on `drain` once every MMA the warp issued has
 // completed, so TMEM is not released under a running MMA.
@@ -584,12 +598,16 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   // kernel are spread across the heads instead of delaying one head's whole share
   const int h = blockIdx.x % p.Hkv, ci = blockIdx.x / p.Hkv;
   uint32_t* counter = ws.sched + h;
+  // the first claim's round trip overlaps the barrier and TMEM setup
+  const uint32_t first = warp == kProducerWarp && lane == 0 ? atomicAdd(counter, 1u) : 0u;
   const Smem s = carve(smem_raw, NRT * 128, p.nstages);
   const uint32_t tmem = setup(s, p.nstages, 1, kTmemSlots, 4);
   volatile int* ab = s.abort_flag;
 
   if (warp == kProducerWarp) {
-    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, counter, true, false, ws.status);
+    if (lane == 0)
+      produce(s, &tm_q, &tm_k, p, h, counter, ws.sched + SGDKV_MAX_KV_HEADS + h, first, false,
+              ws.status);
   } else if (warp == kMmaWarp) {
     const uint32_t leader = elect_one();
     const uint32_t idesc = idesc_bf16(128, kTileKeys);
@@ -687,7 +705,6 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     }
   }
   teardown(tmem);
-  if (threadIdx.x == 0) finish_claims(counter, ws.sched + SGDKV_MAX_KV_HEADS + h, p.cph);
 }
 
 // ---------------------------------------------------------------------------------------
@@ -739,6 +756,7 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.x % p.Hkv;             // heads interleaved, as in pass 1
   uint32_t* counter = ws.sched + 2 * SGDKV_MAX_KV_HEADS + h;
+  const uint32_t first = warp == kProducerWarp && lane == 0 ? atomicAdd(counter, 1u) : 0u;
   const Smem s = carve(smem_raw, p.GW, p.nstages);
   float* lse2 = s.tail;                          // [kMaxRows], negated
   const uint32_t tmem = setup(s, p.nstages, 1, 2, kEpiWarps);
@@ -747,7 +765,9 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   const int nn = p.GW / nch;                     // MMA N
 
   if (warp == kProducerWarp) {
-    if (lane == 0) produce(s, &tm_q, &tm_k, p, h, counter, true, true, ws.status);
+    if (lane == 0)
+      produce(s, &tm_q, &tm_k, p, h, counter, ws.sched + 3 * SGDKV_MAX_KV_HEADS + h, first, true,
+              ws.status);
   } else if (warp == kMmaWarp) {
     const uint32_t leader = elect_one();
     const uint32_t idesc = idesc_bf16(128, nn);
@@ -923,8 +943,6 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     }
   }
   teardown(tmem);
-  if (threadIdx.x == 0)
-    finish_claims(counter, ws.sched + 3 * SGDKV_MAX_KV_HEADS + h, p.cph);
 }
 
 // scores = max-pool over [j - radius, j + radius] (clipped to the row) of the sum of the
