@@ -285,14 +285,18 @@ decode_partial_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* 
 }
 
 // out[h * nq + r][d] = sum_w 2^(m_w - M) o_w[d] / sum_w 2^(m_w - M) l_w over the head's CTA
-// chunks w (zeros for a head without rows).  One block per (head, query row), two global
-// round trips: every partial's (max, sum) is loaded once (up to two per thread) and kept in
-// registers for the block's maximum, the weights 2^(m_w - M) (to shared memory) and the
-// normaliser; then eight groups of 64 threads (one column pair each) sum the weighted
-// partials w = g, g + 8, ... with all of a thread's loads in flight together.
+// chunks w (zeros for a head without rows).  One block per (head, query row), one global
+// round trip: eight groups of 64 threads (one column pair each) take the partials w = g,
+// g + 8, ...; with its column pair of up to kDCombU of them a thread loads the (max, sum) of
+// one of its group's partials, which reach the group through shared memory (a head has at
+// most kDTargetChunks + 1 chunks: one round of loads covers it); each thread folds its
+// partials into a running (max, weighted sums), and the block combines the threads' results
+// against the block's maximum.
 constexpr int kDCombThreads = 512;
 constexpr int kDMaxChunks = 1024;              // >= kDTargetChunks + SGDKV_MAX_KV_HEADS
 constexpr int kDCombGroups = kDCombThreads / 64;
+constexpr int kDCombU = 20;                    // partials per thread and round trip
+static_assert(kDCombGroups * kDCombU >= kDTargetChunks + 1, "one round trip per head");
 
 __device__ __forceinline__ float block_reduce(float v, bool is_max, float* red) {
 #pragma unroll
@@ -311,10 +315,9 @@ __device__ __forceinline__ float block_reduce(float v, bool is_max, float* red) 
 
 __global__ void __launch_bounds__(kDCombThreads)
 decode_combine_kernel(const float* __restrict__ part, DecodeParams p, float* __restrict__ out) {
-  __shared__ float f[kDMaxChunks];
   __shared__ float red[kDCombThreads / 32];
   __shared__ float2 osum[kDCombGroups][kD / 2];
-  static_assert(kDMaxChunks <= 2 * kDCombThreads, "two partials per thread");
+  __shared__ float2 sml[kDCombGroups][kDCombU];   // (max, sum) of a group's partials
   const int h = blockIdx.x / p.nq, r = blockIdx.x % p.nq, tid = threadIdx.x;
   const int w0 = p.wpfx[h], n = min(p.wpfx[h + 1] - w0, kDMaxChunks);
   auto row = [&](int w) { return part + (size_t(w0 + w) * 16 + r) * kDPartStride; };
@@ -324,44 +327,50 @@ decode_combine_kernel(const float* __restrict__ part, DecodeParams p, float* __r
   // launched as a programmatic dependent of the partial kernel: the partials are complete
   // and visible once this returns (a no-op after an ordinary launch)
   asm volatile("griddepcontrol.wait;" ::: "memory");
-  float2 ml[2];
-#pragma unroll
-  for (int k = 0; k < 2; ++k) {
-    const int w = tid + k * kDCombThreads;
-    ml[k] = w < n ? __ldcg(reinterpret_cast<const float2*>(row(w) + kD))
-                  : make_float2(-INFINITY, 0.f);
-  }
-  const float M = block_reduce(fmaxf(ml[0].x, ml[1].x), true, red);
-  float sl = 0.f;
-#pragma unroll
-  for (int k = 0; k < 2; ++k) {
-    const int w = tid + k * kDCombThreads;
-    if (w < n) {
-      const float fw = ml[k].x == -INFINITY ? 0.f : ex2f(ml[k].x - M);
-      f[w] = fw;
-      sl += fw * ml[k].y;
-    }
-  }
-  const float S = block_reduce(sl, false, red);   // its barriers also publish f
   const int grp = tid >> 6, cp = tid & 63;       // column pair 2 cp, 2 cp + 1
+  float mt = -INFINITY, st = 0.f;                // this thread's running max and sum
   float2 o = make_float2(0.f, 0.f);
-  constexpr int kU = 16;
-  for (int w = grp; w < n; w += kDCombGroups * kU) {
-    float2 v[kU];
+  for (int base = 0; base < n; base += kDCombGroups * kDCombU) {
+    const int w = base + grp;
+    // partial w + 8 k of this group: a fixed stride from partial w (one base address)
+    constexpr size_t kStep = size_t(kDCombGroups) * 16 * kDPartStride / 2;   // in float2
+    const float2* pv = reinterpret_cast<const float2*>(part) +
+                       (size_t(w0 + w) * 16 + r) * (kDPartStride / 2) + cp;
+    float2 v[kDCombU];
 #pragma unroll
-    for (int k = 0; k < kU; ++k) {
-      const int wk = w + kDCombGroups * k;
-      v[k] = wk < n ? __ldcg(reinterpret_cast<const float2*>(row(wk)) + cp)
-                    : make_float2(0.f, 0.f);
+    for (int k = 0; k < kDCombU; ++k)
+      v[k] = w + kDCombGroups * k < n ? __ldcg(pv + kStep * k) : make_float2(0.f, 0.f);
+    if (cp < kDCombU) {
+      const int wk = w + kDCombGroups * cp;
+      sml[grp][cp] = wk < n ? __ldcg(reinterpret_cast<const float2*>(row(wk) + kD))
+                            : make_float2(-INFINITY, 0.f);
     }
+    __syncthreads();
+    float mb = mt;
 #pragma unroll
-    for (int k = 0; k < kU; ++k) {
-      const int wk = w + kDCombGroups * k;
-      const float fw = wk < n ? f[wk] : 0.f;
-      o.x += fw * v[k].x;
-      o.y += fw * v[k].y;
+    for (int k = 0; k < kDCombU; ++k) mb = fmaxf(mb, sml[grp][k].x);
+    if (mb != -INFINITY) {
+      const float sc = mt == -INFINITY ? 0.f : ex2f(mt - mb);
+      o.x *= sc;
+      o.y *= sc;
+      st *= sc;
+#pragma unroll
+      for (int k = 0; k < kDCombU; ++k) {
+        const float2 e = sml[grp][k];
+        const float fw = e.x == -INFINITY ? 0.f : ex2f(e.x - mb);
+        o.x += fw * v[k].x;
+        o.y += fw * v[k].y;
+        st += fw * e.y;
+      }
+      mt = mb;
     }
+    __syncthreads();                             // sml is rewritten by the next round
   }
+  const float M = block_reduce(mt, true, red);
+  const float sc = mt == -INFINITY ? 0.f : ex2f(mt - M);
+  o.x *= sc;
+  o.y *= sc;
+  const float S = block_reduce(cp == 0 ? st * sc : 0.f, false, red);   // one sum per group
   osum[grp][cp] = o;
   __syncthreads();
   if (tid < kD / 2) {
