@@ -132,7 +132,8 @@ SGDKV_API size_t sgdkv_workspace_bytes(int32_t Hq, int32_t Hkv, int64_t L, int32
  * scores_out device fp32 [Hkv][L].
  * Reproducibility: the scoring CTAs claim key tiles dynamically, and how each window row's
  * softmax denominator is summed follows the claims, so two calls on the same input agree to
- * within fp32 rounding (relative ~1e-6), not bit for bit.
+ * within fp32 rounding (relative ~1e-6), not bit for bit (sgdkv_score_ex with
+ * SGDKV_SCORE_DETERMINISTIC: bit for bit).
  * Errors: INVALID_ARG, UNSUPPORTED, WORKSPACE, CUDA (launch failure).
  */
 SGDKV_API sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq, int32_t Hkv, int64_t L,
@@ -163,6 +164,14 @@ SGDKV_API sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq,
  * found on the device, records SGDKV_ERR_INVALID_ARG in the workspace status word
  * (sgdkv_last_error) and its head contributes nothing.  SGDKV_SCORE_AGG_IPT_MAX needs
  * W in {16, 32, 48, 64} and G <= 8 (UNSUPPORTED otherwise).
+ * SGDKV_SCORE_DETERMINISTIC (bit 3): bit-reproducible scores.  By default the scoring CTAs
+ * of a KV head claim its key tiles dynamically (the CTAs that start late, while other
+ * kernels hold SMs, take fewer), so each window row's softmax denominator is summed in an
+ * order that varies between calls.  With this bit the first pass gives CTA c of a head the
+ * key tiles c, c + C, c + 2C, ... (C CTAs per head), and every sum of both passes follows a
+ * fixed order: two calls on the same input and device give the same scores bit for bit,
+ * whatever else the GPU runs meanwhile.  The price is load balance: a CTA that starts late
+ * still has its whole share of tiles.
  * Unknown flag bits, or an IPT mode without head_weights: INVALID_ARG.  Other arguments and
  * errors as sgdkv_score.
  */
@@ -172,6 +181,7 @@ SGDKV_API sgdkv_status sgdkv_score(const void* q_win, const void* K, int32_t Hq,
 #define SGDKV_SCORE_AGG_IPT_MEAN (2u << 1)
 #define SGDKV_SCORE_AGG_IPT_ONLY (3u << 1)
 #define SGDKV_SCORE_AGG_MASK (3u << 1)
+#define SGDKV_SCORE_DETERMINISTIC (1u << 3)
 SGDKV_API sgdkv_status sgdkv_score_ex(const void* q_win, const void* K, int32_t Hq, int32_t Hkv,
                                       int64_t L, int32_t d, int32_t W, int32_t pool,
                                       uint32_t flags, const float* head_weights,

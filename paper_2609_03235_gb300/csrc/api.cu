@@ -140,6 +140,10 @@ static constexpr size_t kStaticScratchBytes = size_t(64) << 20;   // 64 MiB per 
 static __device__ __align__(256) uint8_t sgdkv_static_scratch[kStaticScratchBytes];
 
 namespace {
+// Every scoring flag bit sgdkv.h defines.
+constexpr uint32_t kScoreFlags =
+    SGDKV_SCORE_PROXY_QUERY | SGDKV_SCORE_AGG_MASK | SGDKV_SCORE_DETERMINISTIC;
+
 constexpr int kMaxDevices = 64;
 std::mutex g_scratch_mu;
 void* g_scratch_dev[kMaxDevices] = {};
@@ -201,7 +205,7 @@ sgdkv_status check_score_args(const void* q_win, const void* K, int32_t Hq, int3
                               const float* head_weights) {
   if (!q_win || !K) return SGDKV_ERR_INVALID_ARG;
   if (!aligned16(q_win) || !aligned16(K)) return SGDKV_ERR_INVALID_ARG;
-  if (flags & ~(SGDKV_SCORE_PROXY_QUERY | SGDKV_SCORE_AGG_MASK)) return SGDKV_ERR_INVALID_ARG;
+  if (flags & ~kScoreFlags) return SGDKV_ERR_INVALID_ARG;
   const uint32_t agg = flags & SGDKV_SCORE_AGG_MASK;
   if (agg != SGDKV_SCORE_AGG_SUM && !head_weights) return SGDKV_ERR_INVALID_ARG;
   const sgdkv_status s = check_score_shape(Hq, Hkv, L, d, W);
@@ -278,7 +282,7 @@ sgdkv_status sgdkv_pool_raw(const void* workspace, size_t ws_bytes, int32_t Hkv,
   if (Hkv <= 0 || L <= 0) return SGDKV_ERR_INVALID_ARG;
   if (Hkv > SGDKV_MAX_KV_HEADS || int64_t(Hkv) * L >= (int64_t(1) << 31))
     return SGDKV_ERR_UNSUPPORTED;
-  if (flags & ~(SGDKV_SCORE_PROXY_QUERY | SGDKV_SCORE_AGG_MASK)) return SGDKV_ERR_INVALID_ARG;
+  if (flags & ~kScoreFlags) return SGDKV_ERR_INVALID_ARG;
   sgdkv_status s = check_pool(pool);
   if (s != SGDKV_OK) return s;
   if ((s = check_workspace(const_cast<void*>(workspace), ws_bytes, Hkv, L)) != SGDKV_OK) return s;
@@ -359,7 +363,7 @@ sgdkv_status sgdkv_pool_compact(const void* score_workspace, size_t score_ws_byt
   if (d != kD || Hkv > SGDKV_MAX_KV_HEADS || int64_t(Hkv) * L >= (int64_t(1) << 31))
     return SGDKV_ERR_UNSUPPORTED;
   if (!aligned16(K) || !aligned16(V) || !aligned16(scores_out)) return SGDKV_ERR_INVALID_ARG;
-  if (flags & ~(SGDKV_SCORE_PROXY_QUERY | SGDKV_SCORE_AGG_MASK)) return SGDKV_ERR_INVALID_ARG;
+  if (flags & ~kScoreFlags) return SGDKV_ERR_INVALID_ARG;
   sgdkv_status s = check_pool(pool);
   if (s != SGDKV_OK) return s;
   HeadTable ht;

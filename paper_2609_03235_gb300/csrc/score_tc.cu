@@ -73,6 +73,7 @@ struct TcParams {
   int causal;     // 1: window row w sees keys <= L - W + w; 0: every row sees all L keys
   int agg;        // SGDKV_SCORE_AGG_* >> 1: 0 sum over the group, 1 IPT max, 2 IPT mean, 3 IPT only
   const float* head_w;   // IPT modes: summarization score per query head [Hq]
+  int det;        // SGDKV_SCORE_DETERMINISTIC: pass 1 takes fixed key tiles per CTA
   uint64_t wait_ns;
   uint32_t flags;
 };
@@ -433,7 +434,8 @@ __device__ __forceinline__ void finish_claims(uint32_t* counter, uint32_t* finis
 
 // TMA producer (one thread): key tiles of head h claimed one at a time from the head's
 // counter (shared by the head's CTAs; `first` is the claim made at kernel entry, the next
-// claim is made while the current tile's stage is awaited) until none are left, and the Q
+// claim is made while the current tile's stage is awaited) until none are left -- or, with
+// stride > 0, the fixed tiles first, first + stride, ... (no counter) -- and the Q
 // rows of head h once, right after the first key tile (which comes from HBM, the Q rows from
 // L2); the stage after the last tile carries tile id -1 and no data.  Once its last claim
 // has returned the thread counts the CTA's claims finished (finish_claims), while the CTA's
@@ -443,7 +445,7 @@ __device__ __forceinline__ void finish_claims(uint32_t* counter, uint32_t* finis
 // pass 2), so that its misses do not push out the tiles it has yet to reach.
 __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMap* tm_k,
                         const TcParams& p, int h, uint32_t* counter, uint32_t* finished,
-                        uint32_t first, bool second, uint32_t* status) {
+                        uint32_t first, uint32_t stride, bool second, uint32_t* status) {
   volatile int* ab = s.abort_flag;
   bool q_issued = false;
   auto load_q = [&] {
@@ -464,7 +466,7 @@ __device__ void produce(const Smem& s, const CUtensorMap* tm_q, const CUtensorMa
     const uint32_t claim = next;
     const uint32_t tile =
         second && claim < uint32_t(p.T) ? uint32_t(p.T) - 1u - claim : claim;
-    if (claim < uint32_t(p.T)) next = atomicAdd(counter, 1u);
+    if (claim < uint32_t(p.T)) next = stride ? claim + stride : atomicAdd(counter, 1u);
     if (!bwait(bar_kempty(s, st), (use & 1) ^ 1, ab, p.wait_ns, status)) break;
     if (tile >= uint32_t(p.T)) {
       st_tile(s.stile + st, -1);
@@ -598,16 +600,18 @@ score_pass1_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
   // kernel are spread across the heads instead of delaying one head's whole share
   const int h = blockIdx.x % p.Hkv, ci = blockIdx.x / p.Hkv;
   uint32_t* counter = ws.sched + h;
-  // the first claim's round trip overlaps the barrier and TMEM setup
-  const uint32_t first = warp == kProducerWarp && lane == 0 ? atomicAdd(counter, 1u) : 0u;
+  // the first claim's round trip overlaps the barrier and TMEM setup; with fixed tiles
+  // (p.det) CTA ci takes tiles ci, ci + cph, ... and the counter is not used
+  const uint32_t first = p.det ? uint32_t(ci)
+                               : (warp == kProducerWarp && lane == 0 ? atomicAdd(counter, 1u) : 0u);
   const Smem s = carve(smem_raw, NRT * 128, p.nstages);
   const uint32_t tmem = setup(s, p.nstages, 1, kTmemSlots, 4);
   volatile int* ab = s.abort_flag;
 
   if (warp == kProducerWarp) {
     if (lane == 0)
-      produce(s, &tm_q, &tm_k, p, h, counter, ws.sched + SGDKV_MAX_KV_HEADS + h, first, false,
-              ws.status);
+      produce(s, &tm_q, &tm_k, p, h, counter, ws.sched + SGDKV_MAX_KV_HEADS + h, first,
+              p.det ? uint32_t(p.cph) : 0u, false, ws.status);
   } else if (warp == kMmaWarp) {
     const uint32_t leader = elect_one();
     const uint32_t idesc = idesc_bf16(128, kTileKeys);
@@ -766,8 +770,8 @@ score_pass2_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
 
   if (warp == kProducerWarp) {
     if (lane == 0)
-      produce(s, &tm_q, &tm_k, p, h, counter, ws.sched + 3 * SGDKV_MAX_KV_HEADS + h, first, true,
-              ws.status);
+      produce(s, &tm_q, &tm_k, p, h, counter, ws.sched + 3 * SGDKV_MAX_KV_HEADS + h, first, 0u,
+              true, ws.status);
   } else if (warp == kMmaWarp) {
     const uint32_t leader = elect_one();
     const uint32_t idesc = idesc_bf16(128, nn);
@@ -1082,6 +1086,7 @@ cudaError_t launch_passes(const __nv_bfloat16* q, const __nv_bfloat16* K, int Hq
   p.causal = (flags & SGDKV_SCORE_PROXY_QUERY) ? 0 : 1;
   p.agg = int((flags & SGDKV_SCORE_AGG_MASK) >> 1);
   p.head_w = head_weights;
+  p.det = (flags & SGDKV_SCORE_DETERMINISTIC) ? 1 : 0;
   if (p.agg != 0 && !head_weights) return cudaErrorInvalidValue;
   if (p.agg == 1 && (W % 16 != 0 || W > 64 || p.G > 8)) return cudaErrorInvalidValue;
   p.wait_ns = g_score_wait_ns;

@@ -168,6 +168,7 @@ def make_workspace(Hq: int, Hkv: int, L: int, W: int, device="cuda", d: int = 12
 
 SCORE_PROXY_QUERY = 1
 SCORE_AGG_SUM, SCORE_AGG_IPT_MAX, SCORE_AGG_IPT_MEAN, SCORE_AGG_IPT_ONLY = 0, 2, 4, 6
+SCORE_DETERMINISTIC = 8
 
 
 def sgdkv_score(q_win, K, W: int, pool: int, scores_out, workspace, stream=None, flags: int = 0,

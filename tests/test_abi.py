@@ -148,7 +148,8 @@ def test_score_rejects_bad_args_before_device_work():
     # sgdkv_score_ex: unknown flag bits, an IPT mode without weights, unsupported IPT max
     # shapes, then the same checks as sgdkv_score
     ex = L.sgdkv_score_ex
-    assert ex(p, p, 28, 4, 1024, 128, 32, 7, 8, None, p, p, 1 << 30, None) == sg.ERR_INVALID_ARG
+    assert ex(p, p, 28, 4, 1024, 128, 32, 7, 16, None, p, p, 1 << 30, None) == sg.ERR_INVALID_ARG
+    assert ex(p, p, 28, 4, 1024, 128, 32, 7, 1 << 31, None, p, p, 1 << 30, None) == sg.ERR_INVALID_ARG
     assert ex(p, p, 28, 4, 1024, 128, 32, 7, sg.SCORE_AGG_IPT_MAX, None, p, p, 1 << 30,
               None) == sg.ERR_INVALID_ARG
     assert ex(p, p, 36, 4, 1024, 128, 32, 7, sg.SCORE_AGG_IPT_MAX, p, p, p, 1 << 30,
@@ -163,7 +164,7 @@ def test_score_rejects_bad_args_before_device_work():
     raw = L.sgdkv_score_raw
     assert raw(None, p, 28, 4, 1024, 128, 32, 0, None, p, 1 << 30, None) == sg.ERR_INVALID_ARG
     assert raw(p, p, 28, 4, 1024, 64, 32, 0, None, p, 1 << 30, None) == sg.ERR_UNSUPPORTED
-    assert raw(p, p, 28, 4, 1024, 128, 32, 8, None, p, 1 << 30, None) == sg.ERR_INVALID_ARG
+    assert raw(p, p, 28, 4, 1024, 128, 32, 16, None, p, 1 << 30, None) == sg.ERR_INVALID_ARG
     assert raw(p, p, 28, 4, 1024, 128, 32, sg.SCORE_AGG_IPT_MAX, None, p, 1 << 30,
                None) == sg.ERR_INVALID_ARG
     assert raw(p, p, 28, 4, 1024, 128, 32, 0, None, p, 16, None) == sg.ERR_WORKSPACE
@@ -171,14 +172,14 @@ def test_score_rejects_bad_args_before_device_work():
     for fn in (L.sgdkv_window_stats, L.sgdkv_window_sums):
         assert fn(None, p, 28, 4, 1024, 128, 32, 0, None, p, 1 << 30, None) == sg.ERR_INVALID_ARG
         assert fn(p, p, 28, 4, 1024, 64, 32, 0, None, p, 1 << 30, None) == sg.ERR_UNSUPPORTED
-        assert fn(p, p, 28, 4, 1024, 128, 32, 8, None, p, 1 << 30, None) == sg.ERR_INVALID_ARG
+        assert fn(p, p, 28, 4, 1024, 128, 32, 16, None, p, 1 << 30, None) == sg.ERR_INVALID_ARG
         assert fn(p, p, 28, 4, 1024, 128, 32, 0, None, p, 16, None) == sg.ERR_WORKSPACE
     # ...and sgdkv_pool_raw its pool kernel, shape, flags, output and workspace
     pr = L.sgdkv_pool_raw
     assert pr(p, 1 << 30, 4, 1024, 6, 0, p, None) == sg.ERR_INVALID_ARG      # even pool
     assert pr(p, 1 << 30, 0, 1024, 7, 0, p, None) == sg.ERR_INVALID_ARG      # Hkv
     assert pr(p, 1 << 30, 4, 0, 7, 0, p, None) == sg.ERR_INVALID_ARG         # L
-    assert pr(p, 1 << 30, 4, 1024, 7, 8, p, None) == sg.ERR_INVALID_ARG      # unknown flag
+    assert pr(p, 1 << 30, 4, 1024, 7, 16, p, None) == sg.ERR_INVALID_ARG     # unknown flag
     assert pr(p, 1 << 30, 4, 1024, 7, 0, None, None) == sg.ERR_INVALID_ARG   # no output
     assert pr(p, 1 << 30, 99, 1024, 7, 0, p, None) == sg.ERR_UNSUPPORTED     # Hkv > max
     assert pr(p, 16, 4, 1024, 7, 0, p, None) == sg.ERR_WORKSPACE
@@ -192,7 +193,7 @@ def test_score_rejects_bad_args_before_device_work():
                   ws, None)
     assert call(pool=6) == sg.ERR_INVALID_ARG                 # even pool
     assert call(pool=65) == sg.ERR_INVALID_ARG                # window wider than 63
-    assert call(flags=8) == sg.ERR_INVALID_ARG                # unknown flag
+    assert call(flags=16) == sg.ERR_INVALID_ARG               # unknown flag
     assert call(scores=None) == sg.ERR_INVALID_ARG            # pooled scores required
     assert call(d=64) == sg.ERR_UNSUPPORTED                   # head dim
     assert call(budgets=bad) == sg.ERR_INVALID_ARG            # budget above L

@@ -1,0 +1,105 @@
+"""SGDKV_SCORE_DETERMINISTIC: the scores match the oracle and are bit-identical from call to
+call, whatever else runs on the GPU meanwhile.
+
+By default the scoring CTAs claim key tiles dynamically, so the order in which each window
+row's softmax denominator (Section 3.3's window attention) is summed depends on when each
+CTA started.  With the flag the first pass gives every CTA a fixed set of key tiles.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import sgdkv_oracle as O
+from paper_2609_03235_gb300 import configs, synth
+from paper_2609_03235_gb300 import sgdkv as sg
+
+pytestmark = pytest.mark.gpu
+RTOL, ATOL = 2e-3, 1e-5
+SCHED_BYTES = (1024, 2048)     # the scorer's key-tile counters inside the workspace
+
+
+@pytest.fixture(scope="module")
+def dev():
+    sg.lib()
+    return torch.device("cuda:0")
+
+
+def _within(got, exp):
+    return np.abs(got.astype(np.float64) - exp) <= ATOL + RTOL * np.abs(exp.astype(np.float64))
+
+
+CASES = [
+    # Hq, Hkv, L, W, flags name
+    (28, 4, 3000, 64, "sum"),
+    (14, 2, 1000, 32, "proxy"),
+    (28, 4, 20000, 64, "sum"),      # several key tiles per CTA
+    (16, 2, 2049, 64, "ipt_mean"),
+    (28, 4, 129, 64, "sum"),        # fewer key tiles than CTAs per head
+]
+
+
+@pytest.mark.parametrize("Hq,Hkv,L,W,flags_name", CASES)
+def test_deterministic_score_parity(dev, Hq, Hkv, L, W, flags_name):
+    wl = synth.tiny_workload(Hq=Hq, Hkv=Hkv, d=128, L=L, W=W, n_salient=min(8, max(0, L - W - 4)))
+    inp = synth.tiny_inputs(wl, tag=900 + L)
+    q = synth.to_torch_bf16(inp["q"], dev)
+    K = synth.to_torch_bf16(inp["K"], dev)
+    flags = sg.SCORE_DETERMINISTIC
+    hw, causal = None, True
+    if flags_name == "proxy":
+        flags |= sg.SCORE_PROXY_QUERY
+        causal = False
+    w = None
+    if flags_name == "ipt_mean":
+        flags |= sg.SCORE_AGG_IPT_MEAN
+        w = np.random.default_rng(L).random(Hq).astype(np.float32)
+        hw = torch.from_numpy(w).to(dev)
+    ws = sg.make_workspace(Hq, Hkv, L, W, dev)
+    out = torch.empty((Hkv, L), dtype=torch.float32, device=dev)
+    for _ in range(2):
+        sg.sgdkv_score(q, K, W, 7, out, ws, flags=flags, head_weights=hw)
+    torch.cuda.synchronize()
+    assert sg.sgdkv_last_error(ws) == sg.OK
+    assert int(ws[SCHED_BYTES[0]:SCHED_BYTES[1]].count_nonzero()) == 0
+    if w is None:
+        raw = O.window_scores(inp["q"], inp["K"], causal=causal)
+    else:
+        raw = O.window_scores_ipt(inp["q"], inp["K"], w, O.AGG_IPT_MEAN, causal=causal)
+    exp = O.max_pool(raw, 7)
+    got = out.cpu().numpy()
+    ok = _within(got, exp)
+    assert ok.all(), f"{(~ok).sum()} of {ok.size} off; worst {np.max(np.abs(got - exp))}"
+
+
+def test_deterministic_scores_bit_identical_under_load(dev):
+    """One full 128K layer (4 KV heads, W = 64) scored three times with the flag: alone,
+    while a large matrix product holds SMs on another stream, and alone again.  Every call
+    gives the same scores bit for bit, and they match the oracle's."""
+    wl = configs.BY_NAME["c3_qwen25_7b_L128k"]
+    inp = synth.layer_inputs_host(wl, 3)
+    q = synth.to_torch_bf16(inp["q"], dev)
+    K = synth.to_torch_bf16(inp["K"], dev)
+    ws = sg.make_workspace(wl.Hq, wl.Hkv, wl.L, wl.W, dev)
+    outs = [torch.empty((wl.Hkv, wl.L), dtype=torch.float32, device=dev) for _ in range(3)]
+    a = torch.randn((8192, 8192), device=dev).to(torch.bfloat16)
+    side = torch.cuda.Stream(dev)
+    flags = sg.SCORE_DETERMINISTIC
+    torch.cuda.synchronize()
+    sg.sgdkv_score(q, K, wl.W, wl.pool, outs[0], ws, flags=flags)
+    torch.cuda.synchronize()
+    with torch.cuda.stream(side):
+        for _ in range(4):
+            c = a @ a
+    sg.sgdkv_score(q, K, wl.W, wl.pool, outs[1], ws, flags=flags)
+    torch.cuda.synchronize()
+    del c
+    sg.sgdkv_score(q, K, wl.W, wl.pool, outs[2], ws, flags=flags)
+    torch.cuda.synchronize()
+    assert sg.sgdkv_last_error(ws) == sg.OK
+    assert int(ws[SCHED_BYTES[0]:SCHED_BYTES[1]].count_nonzero()) == 0
+    assert torch.equal(outs[0], outs[1])
+    assert torch.equal(outs[0], outs[2])
+    exp = O.max_pool(O.window_scores(inp["q"], inp["K"]), wl.pool)
+    got = outs[0].cpu().numpy()
+    ok = _within(got, exp)
+    assert ok.all(), f"{(~ok).sum()} of {ok.size} off; worst {np.max(np.abs(got - exp))}"
