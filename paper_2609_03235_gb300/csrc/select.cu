@@ -243,12 +243,17 @@ sel_cluster_kernel(const float* __restrict__ scores, HeadTable ht, int csize,
   // register-resident positions p0 .. p0+PER-1 (0 bits outside the slice: never read)
   const int64_t p0 = beg + int64_t(tid) * (PER > 0 ? PER : 1);
   uint32_t u[PER > 0 ? PER : 1];
+  // The first push into a peer's shared memory may only happen once every CTA of the
+  // cluster runs: arrive here, wait after the slice is loaded (long since complete by then).
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
   if constexpr (POOL) {
     pool_slice<PER>(ps, h, L, beg, end, p0, u);
   } else if constexpr (PER > 0) {
 #pragma unroll
     for (int i = 0; i < PER; ++i) u[i] = p0 + i < end ? score_key(__ldg(row + p0 + i)) : 0u;
   }
+
+  asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
 
   uint32_t cand = 0u;                       // PER > 0: bit i = position p0+i is middle
   if constexpr (PER > 0) {
@@ -486,7 +491,9 @@ sel_cluster_kernel(const float* __restrict__ scores, HeadTable ht, int csize,
     cu_out[h] = ht.cu[h];
     if (h == ht.Hkv - 1) cu_out[h + 1] = ht.cu[h + 1];
   }
-  cluster.sync();   // no CTA leaves while a peer may still store into its shared memory
+  // No barrier before leaving: the last stores into a peer's shared memory (the kept
+  // counts) precede the cluster barrier above, so no peer touches this CTA's shared memory
+  // any more.
 }
 
 // Copies kept rows: 16 threads per 256-byte row of K and of V.
