@@ -268,11 +268,9 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
         "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
       : "r"(taddr));
 }
-__device__ __forceinline__ void tmem_wait_ld() {
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
-// The same wait, with the registers of the load it completes passed through it: code that
-// reads them cannot be scheduled above the wait while a later load is still in flight.
+// Waits for this thread's TMEM loads, with the registers of the load it completes passed
+// through it: code that reads them cannot be scheduled above the wait while a later load is
+// still in flight.
 __device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[16]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;"
                : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
