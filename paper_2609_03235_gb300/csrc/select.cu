@@ -607,10 +607,21 @@ cudaError_t launch_select(const float* scores, const HeadTable& ht, int csize,
 // Positions per thread of the selection kernel for rows of length L: slices of up to 32
 // positions per thread stay in registers for the whole kernel (the positions per thread
 // follow from the cluster size that kernel actually runs with); 0: the streaming kernel.
+// Rows short enough for 8 positions per thread on fewer CTAs are selected by clusters of
+// this many CTAs or more (measured on the benchmark's step, 32K rows and 4 KV heads: 16-CTA
+// clusters 783 M, 8-CTA 830 M, 4-CTA 825 M tokens/s/layer; 4K rows: 1-CTA clusters 66 M
+// against 79-80 M).
+constexpr int kMinShortCluster = 8;
+
 template <bool POOL>
 int pick_per(int64_t L, int* csize) {
   auto fits = [&](int per, int cs) { return ceil_div(ceil_div(L, cs), kCThreads) <= per; };
-  if (fits(8, *csize = cluster_size<8, POOL>())) return 8;
+  if (fits(8, *csize = cluster_size<8, POOL>())) {
+    // short rows: the smallest cluster of at least kMinShortCluster CTAs whose slices still
+    // fit (fewer peers to push histograms to, and SMs left to the scoring kernels)
+    while (*csize > kMinShortCluster && fits(8, *csize - 1)) --*csize;
+    return 8;
+  }
   if (fits(16, *csize = cluster_size<16, POOL>())) return 16;
   if (fits(32, *csize = cluster_size<32, POOL>())) return 32;
   *csize = cluster_size<0, false>();
