@@ -458,6 +458,8 @@ def roofs(wl, outs, ms_step, n_layers, peaks):
 # Workloads measured beside the headline by the default run: every configuration the
 # compression step is specified on, the 128K Qwen2.5-7B shape at each of its total budgets.
 SWEEP_STEPS, SWEEP_WARMUP = 5, 3
+SWEEP_MIN_LAYER_STEPS = 112   # timed steps x layers at least this: a one-layer step is ~50 us,
+                              # and five of them would be mostly the timed region's start-up
 
 
 def sweep_cases():
@@ -479,13 +481,14 @@ def run_sweep(args, world, local, dev, peaks, skip):
             continue
         wl = configs.BY_NAME[name]
         r = StepRunner(wl, frac, wl.n_layers, dev)
-        m = r.measure(SWEEP_STEPS, SWEEP_WARMUP, 1, world, local)
+        steps = max(SWEEP_STEPS, -(-SWEEP_MIN_LAYER_STEPS // wl.n_layers))
+        m = r.measure(steps, SWEEP_WARMUP, 1, world, local)
         _, rf = roofs(wl, r.outs, m["ms_max"], r.Ls, peaks)
         tf = pass_flops(wl) / (m["top_us"] * 1e-6) / 1e12
         out[key] = {
             "value": world * wl.L * r.Ls / (m["ms_max"] * 1e-3), "unit": UNIT,
             "us_per_layer": 1e3 * m["ms_max"] / r.Ls, "ms_per_step": m["ms_max"],
-            "n_layers": r.Ls, "steps": SWEEP_STEPS, "warmup": SWEEP_WARMUP,
+            "n_layers": r.Ls, "steps": steps, "warmup": SWEEP_WARMUP,
             "model_shape": "Qwen2.5-7B-1M" if wl.Hkv == 4 else "Qwen3-32B",
             "context_len": wl.L, "window": wl.W, "budget_frac": frac,
             **rf,
