@@ -457,6 +457,7 @@ def roofs(wl, outs, ms_step, n_layers, peaks):
 
 # Workloads measured beside the headline by the default run: every configuration the
 # compression step is specified on, the 128K Qwen2.5-7B shape at each of its total budgets.
+E2E_ROUNDS = 3                # timed rounds of the end-to-end run (median reported)
 SWEEP_STEPS, SWEEP_WARMUP = 5, 3
 SWEEP_MIN_LAYER_STEPS = 112   # timed steps x layers at least this: a one-layer step is ~50 us,
                               # and five of them would be mostly the timed region's start-up
@@ -696,15 +697,18 @@ def run_e2e(args, wl, layers, outs, n_sink, n_recent, dev, world):
         step()
     torch.cuda.synchronize(dev)
     K = args.e2e_steps
-    barrier(world)
-    torch.cuda.synchronize(dev)
-    t0 = time.perf_counter()
-    for _ in range(K):
-        step()
-    torch.cuda.synchronize(dev)
-    dt = (time.perf_counter() - t0) / K
-    barrier(world)
-    dt = max_over_ranks(dt, world)
+    rounds = []          # the host link is shared with other jobs: three rounds, the median
+    for _ in range(E2E_ROUNDS):
+        barrier(world)
+        torch.cuda.synchronize(dev)
+        t0 = time.perf_counter()
+        for _ in range(K):
+            step()
+        torch.cuda.synchronize(dev)
+        dt = (time.perf_counter() - t0) / K
+        barrier(world)
+        rounds.append(max_over_ranks(dt, world))
+    dt = sorted(rounds)[len(rounds) // 2]
     for sl in slots:
         st = sg.sgdkv_last_error(sl["ws"])
         if st != sg.OK:
@@ -713,6 +717,7 @@ def run_e2e(args, wl, layers, outs, n_sink, n_recent, dev, world):
             "d2h_bytes_per_step": int(d2h_bytes),
             "host_read_bytes_per_step": int(host_read_bytes),
             "ms_per_step": dt * 1e3, "steps": K,
+            "rounds_ms_per_step": [x * 1e3 for x in rounds], "of_rounds": "median",
             "overlap": "H2D (q, K) / compute / D2H on three streams, two device slots; V stays "
                        "in pinned host memory and the gather reads only the kept rows"}
 
