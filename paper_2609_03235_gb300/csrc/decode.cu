@@ -455,8 +455,9 @@ cudaError_t launch_decode(const __nv_bfloat16* q, const __nv_bfloat16* Kc,
     note_launches(1);
   }
   {
-    // programmatic dependent launch: the merge blocks are scheduled while the partial
-    // kernel runs (they fit beside its CTAs) and start their work as soon as it completes
+    // programmatic dependent launch: the merge blocks are placed on SMs as soon as there is
+    // room (SMs without a partial CTA, then those the partial CTAs leave) and start their
+    // work as soon as the partial kernel completes
     KernelTimer tc(SGDKV_KERNEL_DECODE, stream);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(unsigned(Hkv * p.nq), 1, 1);
