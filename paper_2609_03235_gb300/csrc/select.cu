@@ -33,12 +33,15 @@ constexpr int kPer = 8;                        // positions per thread per write
 constexpr int kRound = kCThreads * kPer;       // positions per write round
 
 constexpr int kMaxCluster = 16;
+static_assert(64 * kMaxCluster <= kCThreads, "one 16-byte histogram piece per thread");
+static_assert(32 * kCThreads < 65536, "packed 16-bit slice counts");
 
 // Cross-CTA data is pushed: every CTA stores its histogram (and later its counts) into
 // each peer's shared memory, so after the cluster barrier all sums read local memory.
 struct SelShared {
   uint32_t wh[kCWarps][256];              // per-warp histograms (neighbouring keys share bins)
   uint32_t hall[2][kMaxCluster][256];     // histograms of every CTA of the cluster, by rank
+  __align__(16) uint32_t hsum[256];       // this CTA's histogram of the pass
   uint32_t call[kMaxCluster][2];          // (kept non-ties, ties) of every CTA, by rank
   uint32_t s_warp[kCWarps + 1];
   uint32_t bcast[2];
@@ -305,8 +308,13 @@ sel_cluster_kernel(const float* __restrict__ scores, HeadTable ht, int csize,
         uint32_t c = 0;
 #pragma unroll
         for (int w = 0; w < kCWarps; ++w) c += sm.wh[w][tid];
-        for (int r = 0; r < csize; ++r)     // push to every CTA of the cluster
-          *cluster.map_shared_rank(&sm.hall[pass & 1][rank][tid], r) = c;
+        sm.hsum[tid] = c;
+      }
+      __syncthreads();
+      if (tid < 64 * csize) {               // push: one 16-byte quarter-row to one peer each
+        const int r = tid >> 6, qd = tid & 63;
+        const uint4 v = reinterpret_cast<const uint4*>(sm.hsum)[qd];
+        reinterpret_cast<uint4*>(cluster.map_shared_rank(&sm.hall[pass & 1][rank][0], r))[qd] = v;
       }
       cluster.sync();                       // every slice's histogram has arrived
       // thread t < 256 takes bin 255 - t: descending digit order
@@ -354,9 +362,19 @@ sel_cluster_kernel(const float* __restrict__ scores, HeadTable ht, int csize,
       nt += kr.tie(x);
     }
   }
-  uint32_t tot_k, tot_t;
-  const uint32_t my_k_before = block_excl_scan(nk, sm.s_warp, &tot_k);
-  const uint32_t my_t_before = block_excl_scan(nt, sm.s_warp, &tot_t);
+  uint32_t tot_k, tot_t, my_k_before, my_t_before;
+  if constexpr (PER > 0) {
+    // both counts in one scan: a CTA holds at most 32 * 1024 positions, below 2^16
+    uint32_t tot;
+    const uint32_t before = block_excl_scan((nk << 16) | nt, sm.s_warp, &tot);
+    my_k_before = before >> 16;
+    my_t_before = before & 0xffffu;
+    tot_k = tot >> 16;
+    tot_t = tot & 0xffffu;
+  } else {
+    my_k_before = block_excl_scan(nk, sm.s_warp, &tot_k);
+    my_t_before = block_excl_scan(nt, sm.s_warp, &tot_t);
+  }
   if (tid < csize) {                        // push this slice's counts to CTA `tid`
     uint32_t* dst = cluster.map_shared_rank(&sm.call[rank][0], tid);
     dst[0] = tot_k;
