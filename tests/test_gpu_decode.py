@@ -76,6 +76,7 @@ CASES = [
     (8, 1, 2, [5000]),                         # 16 query rows (the most)
     (14, 2, 1, [96, 7000]),                    # uneven heads
     (2, 2, 3, [0, 0]),                         # no rows at all
+    (8, 2, 1, [3, 150000]),                    # one head holds 147 of the 149 chunks
 ]
 
 

@@ -268,6 +268,9 @@ COMPACT_CASES = [
     (1, 600000, 64, 64, "random"),    # streaming selection: several ordered-write rounds
     (8, 5000, 16, 16, "random"),      # 8 x 16 CTAs: the selection copies the rows itself
     (12, 3001, 0, 32, "quarter"),     # the same, ragged slices
+    (3, 80000, 64, 64, "random"),     # 10-CTA clusters (the smallest that holds 8 a thread)
+    (2, 100001, 32, 32, "quarter"),   # 13-CTA clusters, ragged last slice
+    (13, 80000, 16, 16, "random"),    # 13 x 10 CTAs: rows copied inside the selection kernel
 ]
 
 
@@ -380,6 +383,7 @@ POOL_COMPACT_CASES = [
     (2, 1, 300000, 16, 7, "sum"),     # 32 positions per thread
     (2, 1, 600000, 16, 7, "sum"),     # rows too long for register slices: two kernels
     (64, 8, 3000, 32, 7, "sum"),      # 8 KV heads: rows copied inside the selection kernel
+    (28, 4, 72000, 64, 7, "sum"),     # 9-CTA clusters
 ]
 
 
