@@ -103,3 +103,30 @@ def test_deterministic_scores_bit_identical_under_load(dev):
     got = outs[0].cpu().numpy()
     ok = _within(got, exp)
     assert ok.all(), f"{(~ok).sum()} of {ok.size} off; worst {np.max(np.abs(got - exp))}"
+
+
+@pytest.mark.parametrize("flags_name", ["sum", "ipt_max"])
+def test_deterministic_split_passes_equal_one_call(dev, flags_name):
+    """With the flag, the two passes called one at a time (sgdkv_window_stats, then
+    sgdkv_window_sums and sgdkv_pool_raw) give exactly the scores of one sgdkv_score_ex
+    call, and so does a second round; the IPT max aggregation included."""
+    Hq, Hkv, L, W = 28, 4, 30000, 64
+    wl = synth.tiny_workload(Hq=Hq, Hkv=Hkv, d=128, L=L, W=W, n_salient=8)
+    inp = synth.tiny_inputs(wl, tag=950)
+    q = synth.to_torch_bf16(inp["q"], dev)
+    K = synth.to_torch_bf16(inp["K"], dev)
+    flags, hw = sg.SCORE_DETERMINISTIC, None
+    if flags_name == "ipt_max":
+        flags |= sg.SCORE_AGG_IPT_MAX
+        hw = torch.from_numpy(np.random.default_rng(5).random(Hq).astype(np.float32)).to(dev)
+    ws = sg.make_workspace(Hq, Hkv, L, W, dev)
+    one = torch.empty((Hkv, L), dtype=torch.float32, device=dev)
+    sg.sgdkv_score(q, K, W, 7, one, ws, flags=flags, head_weights=hw)
+    for _ in range(2):
+        split = torch.empty((Hkv, L), dtype=torch.float32, device=dev)
+        sg.sgdkv_window_stats(q, K, W, ws, flags=flags, head_weights=hw)
+        sg.sgdkv_window_sums(q, K, W, ws, flags=flags, head_weights=hw)
+        sg.sgdkv_pool_raw(ws, Hkv, L, 7, split, flags=flags)
+        torch.cuda.synchronize()
+        assert sg.sgdkv_last_error(ws) == sg.OK
+        assert torch.equal(one, split)
