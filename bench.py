@@ -48,6 +48,8 @@ def parse_args(argv=None):
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-sweep", action="store_true",
                    help="skip the per-workload measurements beside the headline")
+    p.add_argument("--deterministic", action="store_true",
+                   help="score with SGDKV_SCORE_DETERMINISTIC (bit-reproducible scores)")
     p.add_argument("--no-decode", action="store_true",
                    help="skip the decode-attention measurement over the compressed caches")
     p.add_argument("--cpu-child", action="store_true", help=argparse.SUPPRESS)
@@ -249,7 +251,10 @@ def workload_config(wl, args, world, n_layers):
                        "gather on a second; layer l's pooling and compaction overlap layer "
                        "l+1's scoring",
             "l2": "inputs larger than L2 (K+V of one layer = %d MiB)" %
-                  (2 * wl.Hkv * wl.L * wl.d * 2 >> 20)}
+                  (2 * wl.Hkv * wl.L * wl.d * 2 >> 20),
+            "scores": "bit-reproducible (SGDKV_SCORE_DETERMINISTIC)"
+                      if getattr(args, "deterministic", False) else
+                      "dynamic key-tile claims (reproducible to fp32 rounding)"}
 
 
 
@@ -269,7 +274,7 @@ class StepRunner:
     the allocation still runs on the host every step and must reproduce the budgets the
     graph was captured with."""
 
-    def __init__(self, wl, frac, n_layers, dev):
+    def __init__(self, wl, frac, n_layers, dev, score_flags=0):
         import numpy as np
         import torch
 
@@ -277,6 +282,7 @@ class StepRunner:
         from paper_2609_03235_gb300 import sgdkv as sg
         self.np, self.torch, self.sg = np, torch, sg
         self.wl, self.frac, self.dev = wl, frac, dev
+        self.score_flags = score_flags
         self.n_sink, self.n_recent = configs.sink_recent_split(wl.floor)
         self.hs = synth.head_scores(wl)
         self.T = wl.total_budget(frac)
@@ -314,7 +320,7 @@ class StepRunner:
             wsl = self.ws_score[l % N_SCORE_WS]
             if l >= N_SCORE_WS:
                 s.wait_event(self.pooled[l - N_SCORE_WS])   # its workspace read by then
-            sg.sgdkv_score_raw(inp["q"], inp["K"], wl.W, wsl, s)
+            sg.sgdkv_score_raw(inp["q"], inp["K"], wl.W, wsl, s, flags=self.score_flags)
             self.scored[l].record(s)
             self.sel_stream.wait_event(self.scored[l])
             sg.sgdkv_pool_compact(wsl, wl.pool, inp["K"], inp["V"], o["b"], self.n_sink,
@@ -515,7 +521,8 @@ def run_ours(args, world, rank, local):
     torch.cuda.set_device(dev)
     sg.lib()
     Ls = wl.n_layers if args.layers <= 0 else min(args.layers, wl.n_layers)
-    r = StepRunner(wl, args.frac, Ls, dev)
+    r = StepRunner(wl, args.frac, Ls, dev,
+                   sg.SCORE_DETERMINISTIC if args.deterministic else 0)
     m = r.measure(args.steps, args.warmup, DIAG_STEPS, world, local)
     ms_max = m["ms_max"]
     kern = m["kern"]
